@@ -1,0 +1,457 @@
+"""Slot-decode step benchmark (one layer of Zarya Mode B, Sec. 5.2).
+
+One step = the whole hot path over one batch:
+  stage   zarya_kv_append(STAGE)   the block's K/V -> cache positions P_b..
+  attend  zarya_slot_attn          block rows over prefix + block (mask per sequence)
+  commit  zarya_kv_append(COMMIT)  accepted rows -> cache, P_b += accepted
+then the committed lengths are restored (a 4*B-byte device copy) so every
+step sees the same prefix lengths.
+
+Default workload: decode_small (B8, 16/8 heads, D128, bf16, P=2048,
+contiguous cache, 4 slots x 8 tokens, slot-causal). Inputs are seeded and
+synthetic. Several independent copies of the KV cache rotate so that the
+data touched between two uses of one copy exceeds the L2 cache.
+
+Prints one JSON line. `--impl reference` times the fp64 CPU oracle instead
+(rank 0 only), each step a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+WORKLOAD_LABELS = {
+    "decode_small": "decode_small: B8, Hq16/Hkv8, D128, bf16, prefix 2048, contiguous cache, "
+                    "4 slots x 8 tokens, slot-causal, accept ~U[0,R]",
+    "ragged_mid": "ragged_mid: B32, Hq32/Hkv8, D128, bf16, prefix ~U[512,8192], contiguous, "
+                  "8 slots x 16 tokens, block-bidirectional",
+    "long_ctx": "long_ctx: B4, Hq32/Hkv8, D128, bf16, prefix 32768, contiguous, "
+                "16 slots x 32 tokens, slot-causal",
+    "serving_mix": "serving_mix: B64, Hq32/Hkv8, D128, bf16, paged 16-token pages, prefix "
+                   "log-U[1024,16384], slot_len in {4,8,16,32} x 8 slots, mixed modes",
+}
+
+
+def algorithmic_counts(w):
+    """Bytes / flops the method needs for one step, by the counting rules:
+    K and V of every key a block row can see read once per KV head, Q read
+    once, O written once; 4*D flops per visible (row, head, key) pair;
+    staging and committing move R_b (resp. accepted) rows of K and V, read
+    and written."""
+    eb = 2 if w.dtype == "bf16" else 4
+    P = w.cache_lens.astype(np.int64)
+    R = w.R
+    kv = int((w.Hkv * (P + R) * w.D * eb * 2).sum())
+    qo = int(2 * w.rows * w.Hq * w.D * eb)
+    pairs = 0
+    for b in range(w.B):
+        if w.mask_mode[b] == 0:
+            pairs += w.Hq * int(R[b]) * int(P[b] + R[b])
+        else:
+            pairs += w.Hq * (int(R[b]) * int(P[b]) + int(R[b]) * (int(R[b]) + 1) // 2)
+    row = w.Hkv * w.D * eb
+    return dict(attn_bytes=kv + qo, kv_bytes=kv, flops=4 * w.D * pairs,
+                stage_bytes=int(2 * 2 * R.sum() * row),
+                commit_bytes=int(2 * 2 * w.accept_len.astype(np.int64).sum() * row))
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons."""
+    FIELDS = ("index,timestamp,clocks.sm,clocks.max.sm,power.draw,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def stop(self, t0: float, t1: float):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    ts = time.mktime(time.strptime(parts[1].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                    frac = float("0." + parts[1].split(".")[1]) if "." in parts[1] else 0.0
+                    rows.append((ts + frac, float(parts[2]), float(parts[3]), parts[5:9]))
+                except Exception:
+                    continue
+        inside = [r for r in rows if t0 - 0.05 <= r[0] <= t1 + 0.05]
+        used = inside
+        note = None
+        if not inside and rows:
+            mid = 0.5 * (t0 + t1)
+            used = [min(rows, key=lambda r: abs(r[0] - mid))]
+            note = "timed region shorter than the sampling period: nearest sample"
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in used for i, v in enumerate(r[3]) if v == "Active"})
+        out = {"sm_mhz": float(np.median([r[1] for r in used])) if used else None,
+               "sm_max_mhz": max(r[2] for r in used) if used else None,
+               "reasons": reasons, "samples": len(inside)}
+        if note:
+            out["note"] = note
+        return out
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    if rank == 0:
+        zbuild.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2609_19868_gb300 import _binding as zb
+    from paper_2609_19868_gb300 import session
+    from paper_2609_19868_gb300 import workloads as wl
+
+    zb.load()
+    zb.check_device_error()
+    # weak scaling: every rank runs its own batch (distinct seed)
+    seed = wl.SPECS[args.workload]["seed"] + 1000 * rank
+    w = wl.make(args.workload, seed=seed)
+    if w.both_modes:
+        w = w.with_mode(1)
+    counts = algorithmic_counts(w)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    cache_bytes = (w.k_cache.numel() + w.v_cache.numel()) * w.k_cache.element_size()
+    n_rot = max(2, math.ceil(3 * l2 / max(cache_bytes, 1)))
+    stream = torch.cuda.Stream(dev)
+    rots = []
+    with torch.cuda.stream(stream):
+        base = session.upload(w, dev)
+        rots.append(base)
+        for _ in range(n_rot - 1):
+            kc, vc = base.k_cache.clone(), base.v_cache.clone()
+            db = session.upload(w, dev, caches=(kc, vc))
+            rots.append(db)
+    lens0 = torch.as_tensor(w.cache_lens).to(dev)
+    torch.cuda.synchronize()
+
+    def step(db, ev0=None, ev1=None):
+        db.stage(stream)
+        if ev0 is not None:
+            ev0.record(stream)
+        db.attend(stream)
+        if ev1 is not None:
+            ev1.record(stream)
+        db.commit(stream)
+        db.cache_lens.copy_(lens0, non_blocking=True)
+
+    K, W = args.steps, args.warmup
+    with torch.cuda.stream(stream):
+        for i in range(W):
+            step(rots[i % n_rot])
+    torch.cuda.synchronize()
+    assert zb.check_device_error(stream) == 0
+
+    sampler = ClockSampler(local).start() if args.clocks else None
+    if sampler:
+        time.sleep(0.3)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(K)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(K):
+            step(rots[i % n_rot], *evs[i])
+        end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop(t0, t1) if sampler else None
+    assert zb.check_device_error(stream) == 0
+    total_ms = start.elapsed_time(end)
+    attn_ms = sum(a.elapsed_time(b) for a, b in evs) / K
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    # end to end through the public API: pinned host inputs -> device, the
+    # step, output -> host, every step.
+    q_h = w.q.pin_memory()
+    kn_h = w.k_new.pin_memory()
+    vn_h = w.v_new.pin_memory()
+    acc_h = torch.as_tensor(w.accept_len).pin_memory()
+    out_h = torch.empty_like(w.q).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in (q_h, kn_h, vn_h, acc_h))
+    d2h = out_h.numel() * out_h.element_size()
+
+    def e2e_step(db):
+        db.q.copy_(q_h, non_blocking=True)
+        db.k_new.copy_(kn_h, non_blocking=True)
+        db.v_new.copy_(vn_h, non_blocking=True)
+        db.accept_len.copy_(acc_h, non_blocking=True)
+        step(db)
+        out_h.copy_(db.out, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for i in range(W):
+            e2e_step(rots[i % n_rot])
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for i in range(K):
+            e2e_step(rots[i % n_rot])
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    assert zb.check_device_error(stream) == 0
+
+    hbm_peak, tf_peak, peak_src = read_peaks()
+    attn_gbs = counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9
+    attn_tflops = counts["flops"] / (attn_ms * 1e-3) / 1e12
+    value = K * world / (total_ms * 1e-3)
+    line = {
+        "metric": "slot-decode steps/s (one layer: stage + slot attention + commit)",
+        "value": round(value, 2),
+        "unit": "steps/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(total_ms / K, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1), random-init; no weights or datasets)",
+        "config": {
+            "workload": WORKLOAD_LABELS.get(args.workload, args.workload),
+            "global_batch": w.B * world,
+            "block_rows_per_seq": int(w.max_rows),
+            "kv_len": int((w.cache_lens + w.R).max()),
+            "l2": f"{n_rot} rotating KV caches of {cache_bytes / 1e6:.1f} MB "
+                  f"(> L2 {l2 / 1e6:.0f} MB between reuses)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        },
+        "attn": {
+            "ms_per_launch": round(attn_ms, 5),
+            "hbm_gbs": round(attn_gbs, 1),
+            "tflops": round(attn_tflops, 2),
+            "algorithmic_bytes": counts["attn_bytes"],
+            "algorithmic_flops": counts["flops"],
+        },
+        "roofline": {
+            "bound": "hbm",
+            "achieved": round(attn_gbs, 1),
+            "peak": hbm_peak,
+            "unit": "GB/s",
+            "frac": round(attn_gbs / hbm_peak, 4),
+            "traffic": None,
+            "peak_source": f"{peak_src} HBM copy bandwidth",
+            "kernel": "slot_attn_tc_kernel",
+        },
+        "e2e": {
+            "value": round(K * world / (e2e_ms * 1e-3), 2),
+            "unit": "steps/s",
+            "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h),
+        },
+        "gpu_launches": 4 * K,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _oracle_step(oracle, w, seqs, threads=0):
+    """The oracle's version of one step restricted to sequences ``seqs``."""
+    from dataclasses import replace
+
+    sub = w
+    if len(seqs) < w.B:
+        idx = np.asarray(seqs)
+        offs = w.q_row_offsets
+        rows = np.concatenate([np.arange(offs[b], offs[b + 1]) for b in idx])
+        new_offs = np.concatenate([[0], np.cumsum(w.R[idx])]).astype(np.int32)
+        import torch
+
+        ridx = torch.as_tensor(rows)
+        if w.page_size:
+            raise ValueError("subsets of paged workloads are not used")
+        sub = replace(w, B=len(idx), cache_lens=w.cache_lens[idx], n_slots=w.n_slots[idx],
+                      slot_len=w.slot_len[idx], mask_mode=w.mask_mode[idx],
+                      accept_len=w.accept_len[idx], q_row_offsets=new_offs,
+                      q=w.q[ridx], k_new=w.k_new[ridx], v_new=w.v_new[ridx],
+                      k_cache=w.k_cache[torch.as_tensor(idx)],
+                      v_cache=w.v_cache[torch.as_tensor(idx)])
+    t0 = time.perf_counter()
+    kc, vc, lens = oracle.kv_append(sub.k_new, sub.v_new, sub.R, sub.k_cache, sub.v_cache,
+                                    sub.cache_lens, sub.page_table, sub.q_row_offsets,
+                                    page_size=sub.page_size, commit=False)
+    oracle.slot_attn(sub.q, kc, vc, sub.cache_lens, sub.page_table, sub.n_slots, sub.slot_len,
+                     sub.mask_mode, sub.q_row_offsets, scale=sub.scale,
+                     page_size=sub.page_size, capacity=sub.capacity,
+                     n_pages=sub.n_pages if sub.page_size else -1, threads=threads)
+    oracle.kv_append(sub.k_new, sub.v_new, sub.accept_len, kc, vc, lens, sub.page_table,
+                     sub.q_row_offsets, page_size=sub.page_size, commit=True)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(w, budget_s=20.0):
+    """The oracle, as it stands, on the host cores: whole steps over a subset
+    of the batch's sequences, scaled to the full batch."""
+    import oracle
+
+    oracle.build()
+    cores = oracle.max_threads()
+    t1 = _oracle_step(oracle, w, [0])
+    per_seq = t1
+    n_seq = int(max(1, min(w.B, budget_s / max(per_seq, 1e-6))))
+    t = _oracle_step(oracle, w, list(range(n_seq)))
+    step_s = t * w.B / n_seq
+    return {"value": round(1.0 / step_s, 4), "unit": "steps/s", "cores": cores,
+            "kind": "oracle",
+            "sample": f"{n_seq} of {w.B} sequences of one step (stage + attention + commit, "
+                      f"fp64 C oracle with OpenMP), scaled to the full batch"}
+
+
+def run_reference(args):
+    """The fp64 CPU oracle as the reference arm (rank 0 only)."""
+    world, rank, local = dist_setup()
+    if rank != 0:
+        return
+    import oracle
+    from paper_2609_19868_gb300 import workloads as wl
+
+    oracle.build()
+    w = wl.make(args.workload)
+    if w.both_modes:
+        w = w.with_mode(1)
+    cores = oracle.max_threads()
+    # size each step's sample so the whole run stays within ~2 minutes
+    per_seq = _oracle_step(oracle, w, [0])
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    n_seq = int(max(1, min(w.B, budget / max(per_seq, 1e-6))))
+    for _ in range(args.warmup):
+        _oracle_step(oracle, w, list(range(n_seq)))
+    total = 0.0
+    for _ in range(args.steps):
+        total += _oracle_step(oracle, w, list(range(n_seq)))
+    step_s = total / args.steps * w.B / n_seq
+    value = 1.0 / step_s
+    sample = (f"{n_seq} of {w.B} sequences per step (stage + attention + commit), "
+              f"scaled to the full batch")
+    line = {
+        "impl": "reference",
+        "metric": "slot-decode steps/s (one layer: stage + slot attention + commit)",
+        "value": round(value, 4),
+        "unit": "steps/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_s * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f64",
+        "data": "synthetic (seeded N(0,1), random-init; no weights or datasets)",
+        "config": {"workload": WORKLOAD_LABELS.get(args.workload, args.workload),
+                   "global_batch": w.B},
+        "cpu_baseline": {"value": round(value, 4), "unit": "steps/s", "cores": cores,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="decode_small", choices=list(WORKLOAD_LABELS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
+    ap.add_argument("--no-clocks", dest="clocks", action="store_false")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

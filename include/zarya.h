@@ -1,0 +1,171 @@
+/*
+ * zarya.h -- C ABI of the GB300 (sm_103a) slot-attention library.
+ *
+ * The library implements the per-layer attention step of Zarya's slotted
+ * speculative decoding (Mode B, Sec. 5.2 of "Zarya: A Hybrid
+ * Autoregressive--Masked Diffusion Language Model with Flexible Training and
+ * Dual-Mode Inference") and the KV-cache update with accepted tokens that
+ * gives the mode its full KV reuse (Sec. 5.2 step 7; Sec. 5.1 explains why the
+ * reordered prefix cache stays valid under causal attention).
+ *
+ * Notation: sequence b of a batch of B; committed prefix length
+ * P_b = cache_lens[b]; the current block holds S_b = n_slots[b] slots of
+ * L_b = slot_len[b] tokens, R_b = S_b * L_b query rows, placed right after the
+ * prefix by the reordering step (Sec. 5.2 steps 1-2). Block row r = s*L_b + j
+ * (slot s, offset j). Key index c < P_b is a prefix token; c >= P_b is block
+ * row c - P_b, whose K/V must have been staged into the cache at positions
+ * P_b .. P_b + R_b - 1 (zarya_kv_append with ZARYA_APPEND_STAGE) before
+ * zarya_slot_attn runs.
+ *
+ * General rules for every entry point:
+ *  - All array arguments are DEVICE pointers on the device that owns `stream`
+ *    (the caller owns every buffer). Calls are asynchronous on `stream`; none
+ *    blocks except zarya_check_device_error.
+ *  - Host-side validation happens first; an invalid call returns a status and
+ *    launches nothing. Nothing falls back to the CPU.
+ *  - Errors that only the device can see (a page id out of range, a length
+ *    beyond capacity, inconsistent row offsets, a pipeline wait that timed
+ *    out) set a per-device error word; the affected work is skipped, never
+ *    trapped. Read (and clear) it with zarya_check_device_error.
+ *  - bf16 tensors use round-to-nearest-even on output; fp32 accumulation.
+ */
+#ifndef ZARYA_H_
+#define ZARYA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* zarya_stream_t;
+
+typedef enum {
+  ZARYA_OK = 0,
+  ZARYA_ERR_INVALID_ARG = 1,   /* bad pointer, size, alignment or descriptor field */
+  ZARYA_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement */
+  ZARYA_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed */
+  ZARYA_ERR_DEVICE_FAULT = 4   /* the device error word was set (see below) */
+} zarya_status;
+
+/* Mask of one sequence's block (Sec. 5.2). */
+typedef enum {
+  /* Draft pass (step 3, inter-slot diffusion selection): every block row sees
+   * the whole prefix and the whole block: visible(c) <=> c < P_b + R_b. */
+  ZARYA_MASK_BIDIR_BLOCK = 0,
+  /* Verification pass (step 6, intra-slot autoregressive infilling): causal
+   * over the reordered, flattened sequence: visible(c) <=> c < P_b + r + 1. */
+  ZARYA_MASK_SLOT_CAUSAL = 1
+} zarya_mask_mode;
+
+typedef enum { ZARYA_BF16 = 0, ZARYA_FP32 = 1 } zarya_dtype;
+
+/* zarya_kv_append flags */
+#define ZARYA_APPEND_STAGE 0   /* write rows at P_b.., leave cache_lens unchanged */
+#define ZARYA_APPEND_COMMIT 1  /* write rows at P_b.., then cache_lens[b] += accept_len[b] */
+
+/* Device error word values (zarya_check_device_error's *code). */
+#define ZARYA_DEVERR_NONE 0
+#define ZARYA_DEVERR_PAGE_ID 1        /* page_table entry outside [0, n_pages) */
+#define ZARYA_DEVERR_ROWS 2           /* R_b > max_rows, or q_row_offsets inconsistent with R_b */
+#define ZARYA_DEVERR_CAPACITY 3       /* P_b + rows would pass cache_capacity */
+#define ZARYA_DEVERR_ACCEPT 4         /* accept_len[b] outside [0, R_b] */
+#define ZARYA_DEVERR_TIMEOUT 5        /* a pipeline wait gave up (no progress for ~2 s) */
+#define ZARYA_DEVERR_MASK_MODE 6      /* mask_mode[b] not a zarya_mask_mode */
+
+/* Shapes and host-known bounds shared by both calls. */
+typedef struct {
+  int32_t batch;           /* B >= 1 */
+  int32_t n_q_heads;       /* Hq; Hq % Hkv == 0 (query head h reads KV head h / (Hq/Hkv)) */
+  int32_t n_kv_heads;      /* Hkv */
+  int32_t head_dim;        /* D: 128 for bf16; 32..256 (multiple of 32) for fp32 */
+  int32_t dtype;           /* zarya_dtype of q, caches, k_new/v_new and out */
+  int32_t page_size;       /* 0: contiguous cache [B, cache_capacity, Hkv, D];
+                              else paged cache [n_pages, page_size, Hkv, D] with a page table
+                              [B, cache_capacity / page_size]; bf16 needs 16, 32, 64 or 128 */
+  int32_t cache_capacity;  /* tokens per sequence (paged: max pages per sequence * page_size) */
+  int32_t n_pages;         /* paged: pages in the pool (page ids must lie in [0, n_pages)) */
+  int32_t max_rows;        /* upper bound on R_b over the batch (sizes the grid, no host sync) */
+  int32_t total_rows;      /* rows of q / out / k_new / v_new = q_row_offsets[B] */
+  int32_t max_kv_len;      /* upper bound on P_b + R_b (0: use cache_capacity); sizes splits */
+  int32_t kv_splits;       /* 0: choose automatically; n > 0: split each key range n ways */
+  float scale;             /* softmax scale; 0 means 1 / sqrt(D) */
+  const int32_t* q_row_offsets; /* device [B + 1]: first row of sequence b in q / out /
+                                   k_new; q_row_offsets[b+1] - q_row_offsets[b] == R_b */
+} zarya_attn_desc;
+
+/*
+ * Bytes of scratch memory zarya_slot_attn needs for `desc` (0 if it needs
+ * none). The workspace holds split-KV partial results and per-tile arrival
+ * counters. It must be zero-filled once before its first use; every call
+ * leaves the counters at zero again, so it can be reused by later calls on
+ * the same stream. After a call that set the device error word, zero it again.
+ * Returns 0 as well when desc is invalid (zarya_slot_attn will reject it).
+ */
+size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc);
+
+/*
+ * Slot attention (Sec. 5.2 steps 3 and 6): for every sequence b, query head
+ * h and block row r < R_b,
+ *   out[q_row_offsets[b] + r, h, :] =
+ *     sum_{c visible} softmax_c(scale * q[q_row_offsets[b] + r, h, :] . k_c) v_c
+ * with k_c / v_c the cache entries of token c of sequence b at KV head
+ * h / (Hq / Hkv), and visibility given by mask_mode[b] (zarya_mask_mode).
+ *
+ *  q          [total_rows, Hq, D]                     (read)
+ *  k_cache,   contiguous [B, cache_capacity, Hkv, D]  (read; positions
+ *  v_cache    or paged [n_pages, page_size, Hkv, D]    0 .. P_b + R_b - 1 used)
+ *  cache_lens [B] int32: P_b, the committed prefix (block K/V already staged after it)
+ *  page_table [B, cache_capacity / page_size] int32, or NULL for a contiguous cache
+ *  n_slots, slot_len, mask_mode: [B] int32 each
+ *  out        [total_rows, Hq, D]                     (written; rows of each
+ *                                                      sequence only)
+ *  workspace  zarya_slot_attn_workspace_size(desc) bytes (may be NULL when that is 0)
+ * Pointers q, caches and out must be 16-byte aligned. q/out rows that belong
+ * to no sequence are not written.
+ */
+zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* cache_lens, const int32_t* page_table,
+                             const int32_t* n_slots, const int32_t* slot_len,
+                             const int32_t* mask_mode, void* out, void* workspace,
+                             size_t workspace_bytes, const zarya_attn_desc* desc,
+                             zarya_stream_t stream);
+
+/*
+ * KV-cache update with accepted tokens (Sec. 5.2 step 7): for every sequence
+ * b and i < accept_len[b], row q_row_offsets[b] + i of k_new / v_new
+ * ([total_rows, Hkv, D], the block rows in reordered order, accepted tokens
+ * first) is copied bit for bit to cache position P_b + i (through the page
+ * table when paged). With ZARYA_APPEND_COMMIT, cache_lens[b] then advances by
+ * accept_len[b]; with ZARYA_APPEND_STAGE it is left alone (used to stage a
+ * block's own K/V before its attention pass). 0 <= accept_len[b] <= R_b and
+ * P_b + accept_len[b] <= cache_capacity are checked on the device; a sequence
+ * that fails is skipped and the error word set. Nothing else in the caches
+ * changes.
+ */
+zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
+                             void* k_cache, void* v_cache, int32_t* cache_lens,
+                             const int32_t* page_table, int32_t flags,
+                             const zarya_attn_desc* desc, zarya_stream_t stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the error word of the device
+ * that owns it. Returns ZARYA_OK when it was clear, ZARYA_ERR_DEVICE_FAULT
+ * when it was set (*code receives its ZARYA_DEVERR_* value; code may be
+ * NULL), ZARYA_ERR_CUDA when the synchronisation itself failed.
+ */
+zarya_status zarya_check_device_error(zarya_stream_t stream, int32_t* code);
+
+/* Static, human-readable name of a status. */
+const char* zarya_status_string(zarya_status status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int32_t zarya_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ZARYA_H_ */

@@ -1,0 +1,182 @@
+"""ctypes binding of ``libzarya.so`` (include/zarya.h).
+
+Argument marshalling only: every step of slot attention and KV append runs
+in the library's CUDA kernels. PyTorch supplies device memory and streams.
+If the library is missing the calls raise; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libzarya.so")
+HEADER = os.path.join(os.path.dirname(_PKG), "include", "zarya.h")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_DEVICE_FAULT = 0, 1, 2, 3, 4
+MASK_BIDIR_BLOCK, MASK_SLOT_CAUSAL = 0, 1
+BF16, FP32 = 0, 1
+APPEND_STAGE, APPEND_COMMIT = 0, 1
+DEVERR_NAMES = {0: "none", 1: "page id", 2: "rows", 3: "capacity", 4: "accept length",
+                5: "timeout", 6: "mask mode"}
+
+
+class ZaryaError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {status_string(status)} (status {status})")
+        self.status = status
+
+
+class AttnDesc(ctypes.Structure):
+    """Mirror of ``zarya_attn_desc``."""
+    _fields_ = [
+        ("batch", ctypes.c_int32),
+        ("n_q_heads", ctypes.c_int32),
+        ("n_kv_heads", ctypes.c_int32),
+        ("head_dim", ctypes.c_int32),
+        ("dtype", ctypes.c_int32),
+        ("page_size", ctypes.c_int32),
+        ("cache_capacity", ctypes.c_int32),
+        ("n_pages", ctypes.c_int32),
+        ("max_rows", ctypes.c_int32),
+        ("total_rows", ctypes.c_int32),
+        ("max_kv_len", ctypes.c_int32),
+        ("kv_splits", ctypes.c_int32),
+        ("scale", ctypes.c_float),
+        ("q_row_offsets", ctypes.c_void_p),
+    ]
+
+
+_lib = None
+
+
+def load() -> ctypes.CDLL:
+    """Load the library (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing; build it with __graft_entry__.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    dp = ctypes.POINTER(AttnDesc)
+    lib.zarya_slot_attn_workspace_size.argtypes = [dp]
+    lib.zarya_slot_attn_workspace_size.restype = sz
+    lib.zarya_slot_attn.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, dp, vp]
+    lib.zarya_slot_attn.restype = ctypes.c_int
+    lib.zarya_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, dp, vp]
+    lib.zarya_kv_append.restype = ctypes.c_int
+    lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
+    lib.zarya_check_device_error.restype = ctypes.c_int
+    lib.zarya_status_string.argtypes = [ctypes.c_int]
+    lib.zarya_status_string.restype = ctypes.c_char_p
+    lib.zarya_version.argtypes = []
+    lib.zarya_version.restype = i32
+    _lib = lib
+    return lib
+
+
+def header_functions() -> list:
+    """Names of the functions ``include/zarya.h`` declares."""
+    with open(HEADER) as f:
+        text = f.read()
+    return sorted(set(re.findall(r"\b(zarya_[a-z0-9_]+)\s*\(", text)))
+
+
+def status_string(status: int) -> str:
+    return load().zarya_status_string(int(status)).decode()
+
+
+def version() -> int:
+    return int(load().zarya_version())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check_cuda(name: str, t: torch.Tensor, dtype=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+
+
+def make_desc(*, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int, dtype: int,
+              page_size: int, cache_capacity: int, n_pages: int, max_rows: int,
+              total_rows: int, q_row_offsets: torch.Tensor, max_kv_len: int = 0,
+              kv_splits: int = 0, scale: float = 0.0) -> AttnDesc:
+    _check_cuda("q_row_offsets", q_row_offsets, torch.int32)
+    d = AttnDesc()
+    d.batch, d.n_q_heads, d.n_kv_heads, d.head_dim = batch, n_q_heads, n_kv_heads, head_dim
+    d.dtype, d.page_size, d.cache_capacity, d.n_pages = dtype, page_size, cache_capacity, n_pages
+    d.max_rows, d.total_rows, d.max_kv_len, d.kv_splits = max_rows, total_rows, max_kv_len, kv_splits
+    d.scale = scale
+    d.q_row_offsets = q_row_offsets.data_ptr()
+    d._keep = q_row_offsets  # keep the offsets alive as long as the descriptor
+    return d
+
+
+def workspace_size(desc: AttnDesc) -> int:
+    return int(load().zarya_slot_attn_workspace_size(ctypes.byref(desc)))
+
+
+def slot_attn(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len, mask_mode, out,
+              desc: AttnDesc, workspace: Optional[torch.Tensor] = None, stream=None) -> None:
+    """``zarya_slot_attn``: out <- slot attention of q over the cache (Sec. 5.2)."""
+    for name, t in (("q", q), ("k_cache", k_cache), ("v_cache", v_cache), ("out", out)):
+        _check_cuda(name, t)
+    for name, t in (("cache_lens", cache_lens), ("n_slots", n_slots), ("slot_len", slot_len),
+                    ("mask_mode", mask_mode)):
+        _check_cuda(name, t, torch.int32)
+    if page_table is not None:
+        _check_cuda("page_table", page_table, torch.int32)
+    ws_bytes = 0
+    if workspace is not None:
+        _check_cuda("workspace", workspace)
+        ws_bytes = workspace.numel() * workspace.element_size()
+    st = load().zarya_slot_attn(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_lens),
+                                _ptr(page_table), _ptr(n_slots), _ptr(slot_len),
+                                _ptr(mask_mode), _ptr(out), _ptr(workspace), ws_bytes,
+                                ctypes.byref(desc), _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_slot_attn")
+
+
+def kv_append(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, page_table,
+              desc: AttnDesc, commit: bool = True, stream=None) -> None:
+    """``zarya_kv_append``: copy accepted rows into the cache (Sec. 5.2 step 7)."""
+    for name, t in (("k_new", k_new), ("v_new", v_new), ("k_cache", k_cache),
+                    ("v_cache", v_cache)):
+        _check_cuda(name, t)
+    _check_cuda("accept_len", accept_len, torch.int32)
+    _check_cuda("cache_lens", cache_lens, torch.int32)
+    if page_table is not None:
+        _check_cuda("page_table", page_table, torch.int32)
+    st = load().zarya_kv_append(_ptr(k_new), _ptr(v_new), _ptr(accept_len), _ptr(k_cache),
+                                _ptr(v_cache), _ptr(cache_lens), _ptr(page_table),
+                                APPEND_COMMIT if commit else APPEND_STAGE, ctypes.byref(desc),
+                                _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_kv_append")
+
+
+def check_device_error(stream=None) -> int:
+    """Synchronise and return (and clear) the device error word (0 = none)."""
+    code = ctypes.c_int32(0)
+    st = load().zarya_check_device_error(_stream(stream), ctypes.byref(code))
+    if st not in (OK, ERR_DEVICE_FAULT):
+        raise ZaryaError(st, "zarya_check_device_error")
+    return int(code.value)

@@ -1,0 +1,384 @@
+// Host side of the C ABI declared in include/zarya.h: argument validation,
+// device selection, TMA tensor-map encoding, split planning, workspace
+// layout and kernel launches. Allocates nothing.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "internal.cuh"
+
+namespace zarya {
+namespace {
+
+constexpr int32_t kVersion = 100;  // 0.1.0
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Makes the device that owns `stream` (or, for the legacy default stream, the
+// device that owns `ptr`) current for this thread.
+cudaError_t select_device(cudaStream_t stream, const void* ptr) {
+  int want = -1;
+  if (stream != nullptr) {
+    cudaError_t e = cudaStreamGetDevice(stream, &want);
+    if (e != cudaSuccess) return e;
+  } else {
+    cudaPointerAttributes attr{};
+    cudaError_t e = cudaPointerGetAttributes(&attr, ptr);
+    if (e != cudaSuccess) return e;
+    if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
+      return cudaErrorInvalidValue;
+    want = attr.device;
+  }
+  int cur = -1;
+  cudaError_t e = cudaGetDevice(&cur);
+  if (e != cudaSuccess) return e;
+  if (cur != want) return cudaSetDevice(want);
+  return cudaSuccess;
+}
+
+int sm_count() {
+  constexpr int kMaxDevices = 64;
+  static int cache[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 148;
+  int n = __atomic_load_n(&cache[dev], __ATOMIC_ACQUIRE);
+  if (n == 0) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 148;
+    __atomic_store_n(&cache[dev], n, __ATOMIC_RELEASE);
+  }
+  return n;
+}
+
+zarya_status check_desc(const zarya_attn_desc* d) {
+  if (d == nullptr) return ZARYA_ERR_INVALID_ARG;
+  if (d->batch < 1 || d->n_q_heads < 1 || d->n_kv_heads < 1 || d->head_dim < 1)
+    return ZARYA_ERR_INVALID_ARG;
+  if (d->n_q_heads % d->n_kv_heads != 0) return ZARYA_ERR_INVALID_ARG;
+  if (d->dtype != ZARYA_BF16 && d->dtype != ZARYA_FP32) return ZARYA_ERR_INVALID_ARG;
+  if (d->page_size < 0 || d->cache_capacity < 1 || d->max_rows < 1 || d->total_rows < 1 ||
+      d->max_kv_len < 0 || d->kv_splits < 0 || d->n_pages < 0)
+    return ZARYA_ERR_INVALID_ARG;
+  if (!(d->scale >= 0.f) || std::isinf(d->scale)) return ZARYA_ERR_INVALID_ARG;
+  if (d->q_row_offsets == nullptr) return ZARYA_ERR_INVALID_ARG;
+  if (d->page_size > 0) {
+    if (d->cache_capacity % d->page_size != 0 || d->n_pages < 1) return ZARYA_ERR_INVALID_ARG;
+  }
+  if (static_cast<long long>(d->batch) * d->cache_capacity > 0x7fffffffLL &&
+      d->page_size == 0)
+    return ZARYA_ERR_UNSUPPORTED;
+  const int eb = d->dtype == ZARYA_BF16 ? 2 : 4;
+  if ((static_cast<long long>(d->n_kv_heads) * d->head_dim * eb) % 16 != 0)
+    return ZARYA_ERR_UNSUPPORTED;
+  return ZARYA_OK;
+}
+
+// Attention-specific support checks.
+zarya_status check_attn_support(const zarya_attn_desc* d) {
+  if (d->dtype == ZARYA_BF16) {
+    if (d->head_dim != kHeadDim) return ZARYA_ERR_UNSUPPORTED;
+    const int g = d->n_q_heads / d->n_kv_heads;
+    if (g > kBlockM || kBlockM % g != 0) return ZARYA_ERR_UNSUPPORTED;
+    if (d->page_size != 0 && d->page_size != 16 && d->page_size != 32 && d->page_size != 64 &&
+        d->page_size != 128)
+      return ZARYA_ERR_UNSUPPORTED;
+  } else {
+    if (d->head_dim % 32 != 0 || d->head_dim > 256) return ZARYA_ERR_UNSUPPORTED;
+  }
+  return ZARYA_OK;
+}
+
+struct Plan {
+  int g, m_tiles, splits;
+  long long units;
+  size_t off_lse, off_cnt, bytes;
+};
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// Split-KV plan of the tensor-core path. Work tiles (sequence, KV head,
+// M-tile) whose count already fills the GPU run unsplit; otherwise the key
+// range of each is split so that the slowest CTA (waves x tiles per CTA,
+// plus a fixed per-CTA cost) is as short as possible.
+Plan plan_tc(const zarya_attn_desc* d, int sms) {
+  Plan p{};
+  p.g = d->n_q_heads / d->n_kv_heads;
+  p.m_tiles = static_cast<int>((static_cast<long long>(d->max_rows) * p.g + kBlockM - 1) / kBlockM);
+  p.units = static_cast<long long>(d->batch) * d->n_kv_heads * p.m_tiles;
+  const long long kv_max = d->max_kv_len > 0 ? d->max_kv_len : d->cache_capacity;
+  const int tiles = static_cast<int>((kv_max + kBlockN - 1) / kBlockN);
+  int splits = 1;
+  if (d->kv_splits > 0) {
+    splits = d->kv_splits < tiles ? d->kv_splits : tiles;
+  } else if (p.units < sms) {
+    double best = 1e30;
+    for (int s = 1; s <= tiles && s <= 32; ++s) {
+      const long long waves = (p.units * s + sms - 1) / sms;
+      const double cost = static_cast<double>(waves) * ((tiles + s - 1) / s + 2.0) +
+                          (s > 1 ? 1.0 : 0.0);
+      if (cost < best - 1e-9) {
+        best = cost;
+        splits = s;
+      }
+    }
+  }
+  if (splits < 1) splits = 1;
+  p.splits = splits;
+  if (splits > 1) {
+    const size_t n = static_cast<size_t>(p.units) * splits * kBlockM;
+    const size_t bytes_o = n * kHeadDim * sizeof(float);
+    p.off_lse = align256(bytes_o);
+    p.off_cnt = align256(p.off_lse + n * sizeof(float));
+    p.bytes = align256(p.off_cnt + static_cast<size_t>(p.units) * sizeof(int32_t));
+  }
+  return p;
+}
+
+CUresult encode(CUtensorMap* map, void* base, cuuint32_t rank, const cuuint64_t* dims,
+                const cuuint64_t* strides, const cuuint32_t* box) {
+  auto fn = tensor_map_encoder();
+  if (fn == nullptr) return CUDA_ERROR_NOT_FOUND;
+  const cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, base, dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+}  // namespace
+}  // namespace zarya
+
+using namespace zarya;
+
+extern "C" {
+
+size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc) {
+  if (check_desc(desc) != ZARYA_OK || check_attn_support(desc) != ZARYA_OK) return 0;
+  if (desc->dtype != ZARYA_BF16) return 0;
+  return plan_tc(desc, sm_count()).bytes;
+}
+
+zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* cache_lens, const int32_t* page_table,
+                             const int32_t* n_slots, const int32_t* slot_len,
+                             const int32_t* mask_mode, void* out, void* workspace,
+                             size_t workspace_bytes, const zarya_attn_desc* desc,
+                             zarya_stream_t stream_) {
+  zarya_status st = check_desc(desc);
+  if (st != ZARYA_OK) return st;
+  st = check_attn_support(desc);
+  if (st != ZARYA_OK) return st;
+  if (!q || !k_cache || !v_cache || !cache_lens || !n_slots || !slot_len || !mask_mode || !out)
+    return ZARYA_ERR_INVALID_ARG;
+  if ((desc->page_size > 0) != (page_table != nullptr)) return ZARYA_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
+    return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  if (select_device(stream, q) != cudaSuccess) return ZARYA_ERR_CUDA;
+  cudaError_t ce = cudaSuccess;
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return ZARYA_ERR_CUDA;
+  const float scale =
+      desc->scale > 0.f ? desc->scale : 1.0f / std::sqrt(static_cast<float>(desc->head_dim));
+  const int max_pages = desc->page_size > 0 ? desc->cache_capacity / desc->page_size : 0;
+
+  if (desc->dtype == ZARYA_FP32) {
+    SimtParams p{};
+    p.q = q;
+    p.k_cache = k_cache;
+    p.v_cache = v_cache;
+    p.cache_lens = cache_lens;
+    p.page_table = page_table;
+    p.n_slots = n_slots;
+    p.slot_len = slot_len;
+    p.mask_mode = mask_mode;
+    p.q_row_offsets = desc->q_row_offsets;
+    p.out = out;
+    p.err = err;
+    p.B = desc->batch;
+    p.Hq = desc->n_q_heads;
+    p.Hkv = desc->n_kv_heads;
+    p.D = desc->head_dim;
+    p.max_rows = desc->max_rows;
+    p.total_rows = desc->total_rows;
+    p.capacity = desc->cache_capacity;
+    p.page_size = desc->page_size;
+    p.max_pages = max_pages;
+    p.n_pages = desc->n_pages;
+    p.scale = scale;
+    return launch_slot_attn_f32(p, stream) == cudaSuccess ? ZARYA_OK : ZARYA_ERR_CUDA;
+  }
+
+  const Plan plan = plan_tc(desc, sm_count());
+  if (plan.units > 0x7fffffffLL || plan.m_tiles > 0x7fffffff ||
+      static_cast<long long>(desc->batch) * desc->n_kv_heads > 65535 || plan.splits > 65535)
+    return ZARYA_ERR_UNSUPPORTED;
+  if (plan.bytes > 0) {
+    if (workspace == nullptr || workspace_bytes < plan.bytes ||
+        (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+      return ZARYA_ERR_INVALID_ARG;
+  }
+
+  const int D = desc->head_dim, Hq = desc->n_q_heads, Hkv = desc->n_kv_heads, g = plan.g;
+  CUtensorMap map_q, map_k, map_v;
+  {
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(Hq),
+                                static_cast<cuuint64_t>(desc->total_rows)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2,
+                                   static_cast<cuuint64_t>(Hq) * D * 2};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(g),
+                               static_cast<cuuint32_t>(kBlockM / g)};
+    if (encode(&map_q, const_cast<void*>(q), 3, dims, strides, box) != CUDA_SUCCESS)
+      return ZARYA_ERR_CUDA;
+  }
+  {
+    cuuint64_t dims[4], strides[3];
+    cuuint32_t box[4];
+    dims[0] = D;
+    dims[1] = Hkv;
+    strides[0] = static_cast<cuuint64_t>(D) * 2;
+    strides[1] = static_cast<cuuint64_t>(Hkv) * D * 2;
+    box[0] = 64;
+    box[1] = 1;
+    box[3] = 1;
+    if (desc->page_size == 0) {
+      dims[2] = desc->cache_capacity;
+      dims[3] = desc->batch;
+      strides[2] = static_cast<cuuint64_t>(desc->cache_capacity) * Hkv * D * 2;
+      box[2] = kBlockN;
+    } else {
+      dims[2] = desc->page_size;
+      dims[3] = desc->n_pages;
+      strides[2] = static_cast<cuuint64_t>(desc->page_size) * Hkv * D * 2;
+      box[2] = desc->page_size;
+    }
+    if (encode(&map_k, const_cast<void*>(k_cache), 4, dims, strides, box) != CUDA_SUCCESS ||
+        encode(&map_v, const_cast<void*>(v_cache), 4, dims, strides, box) != CUDA_SUCCESS)
+      return ZARYA_ERR_CUDA;
+  }
+
+  TcParams p{};
+  p.cache_lens = cache_lens;
+  p.page_table = page_table;
+  p.n_slots = n_slots;
+  p.slot_len = slot_len;
+  p.mask_mode = mask_mode;
+  p.q_row_offsets = desc->q_row_offsets;
+  p.out = out;
+  if (plan.bytes > 0) {
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    p.ws_o = reinterpret_cast<float*>(ws);
+    p.ws_lse = reinterpret_cast<float*>(ws + plan.off_lse);
+    p.ws_count = reinterpret_cast<int32_t*>(ws + plan.off_cnt);
+  }
+  p.err = err;
+  p.B = desc->batch;
+  p.Hq = Hq;
+  p.Hkv = Hkv;
+  p.g = g;
+  p.max_rows = desc->max_rows;
+  p.total_rows = desc->total_rows;
+  p.capacity = desc->cache_capacity;
+  p.page_size = desc->page_size;
+  p.max_pages = max_pages;
+  p.n_pages = desc->n_pages;
+  p.m_tiles = plan.m_tiles;
+  p.splits = plan.splits;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  return launch_slot_attn_tc(map_q, map_k, map_v, p, stream) == cudaSuccess ? ZARYA_OK
+                                                                           : ZARYA_ERR_CUDA;
+}
+
+zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
+                             void* k_cache, void* v_cache, int32_t* cache_lens,
+                             const int32_t* page_table, int32_t flags,
+                             const zarya_attn_desc* desc, zarya_stream_t stream_) {
+  zarya_status st = check_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (flags != ZARYA_APPEND_STAGE && flags != ZARYA_APPEND_COMMIT) return ZARYA_ERR_INVALID_ARG;
+  if (!k_new || !v_new || !accept_len || !k_cache || !v_cache || !cache_lens)
+    return ZARYA_ERR_INVALID_ARG;
+  if ((desc->page_size > 0) != (page_table != nullptr)) return ZARYA_ERR_INVALID_ARG;
+  if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
+    return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  if (select_device(stream, k_new) != cudaSuccess) return ZARYA_ERR_CUDA;
+  cudaError_t ce = cudaSuccess;
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return ZARYA_ERR_CUDA;
+  const int eb = desc->dtype == ZARYA_BF16 ? 2 : 4;
+  AppendParams p{};
+  p.k_new = k_new;
+  p.v_new = v_new;
+  p.accept_len = accept_len;
+  p.k_cache = k_cache;
+  p.v_cache = v_cache;
+  p.cache_lens = cache_lens;
+  p.page_table = page_table;
+  p.q_row_offsets = desc->q_row_offsets;
+  p.err = err;
+  p.B = desc->batch;
+  p.row_bytes = desc->n_kv_heads * desc->head_dim * eb;
+  p.max_rows = desc->max_rows;
+  p.total_rows = desc->total_rows;
+  p.capacity = desc->cache_capacity;
+  p.page_size = desc->page_size;
+  p.max_pages = desc->page_size > 0 ? desc->cache_capacity / desc->page_size : 0;
+  p.n_pages = desc->n_pages;
+  if (desc->batch > 65535) return ZARYA_ERR_UNSUPPORTED;
+  return launch_kv_append(p, flags == ZARYA_APPEND_COMMIT, stream) == cudaSuccess
+             ? ZARYA_OK
+             : ZARYA_ERR_CUDA;
+}
+
+zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {
+  if (code) *code = 0;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  if (stream != nullptr) {
+    int dev = -1, cur = -1;
+    if (cudaStreamGetDevice(stream, &dev) != cudaSuccess) return ZARYA_ERR_CUDA;
+    if (cudaGetDevice(&cur) != cudaSuccess) return ZARYA_ERR_CUDA;
+    if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return ZARYA_ERR_CUDA;
+  }
+  cudaError_t ce = cudaSuccess;
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return ZARYA_ERR_CUDA;
+  int host = 0;
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return ZARYA_ERR_CUDA;
+  if (cudaMemcpyAsync(&host, err, sizeof(int), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+    return ZARYA_ERR_CUDA;
+  if (cudaMemsetAsync(err, 0, sizeof(int), stream) != cudaSuccess) return ZARYA_ERR_CUDA;
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return ZARYA_ERR_CUDA;
+  if (code) *code = host;
+  return host == 0 ? ZARYA_OK : ZARYA_ERR_DEVICE_FAULT;
+}
+
+const char* zarya_status_string(zarya_status status) {
+  switch (status) {
+    case ZARYA_OK: return "ok";
+    case ZARYA_ERR_INVALID_ARG: return "invalid argument";
+    case ZARYA_ERR_UNSUPPORTED: return "unsupported configuration";
+    case ZARYA_ERR_CUDA: return "CUDA error";
+    case ZARYA_ERR_DEVICE_FAULT: return "device error word set";
+  }
+  return "unknown status";
+}
+
+int32_t zarya_version(void) { return kVersion; }
+
+}  // extern "C"

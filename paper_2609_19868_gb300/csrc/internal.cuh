@@ -1,0 +1,90 @@
+// Internal declarations shared by the library's translation units: kernel
+// parameter blocks, launchers and the per-device error word.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "zarya.h"
+
+namespace zarya {
+
+// Tile geometry of the tensor-core path (bf16, D = 128).
+constexpr int kBlockM = 128;  // packed (block row, query head) rows per CTA
+constexpr int kBlockN = 128;  // keys per pipeline tile
+constexpr int kHeadDim = 128;
+
+// Parameters of the tensor-core slot-attention kernel (tensor maps travel as
+// separate __grid_constant__ arguments).
+struct TcParams {
+  const int32_t* cache_lens;
+  const int32_t* page_table;
+  const int32_t* n_slots;
+  const int32_t* slot_len;
+  const int32_t* mask_mode;
+  const int32_t* q_row_offsets;
+  void* out;          // bf16 [total_rows, Hq, D]
+  float* ws_o;        // [units, splits, kBlockM, D] fp32 partial outputs (normalised)
+  float* ws_lse;      // [units, splits, kBlockM] log2-sum-exp of each partial
+  int32_t* ws_count;  // [units] arrival counters (zero between calls)
+  int* err;           // device error word
+  int B, Hq, Hkv, g;
+  int max_rows, total_rows, capacity;
+  int page_size, max_pages, n_pages;
+  int m_tiles, splits;
+  float scale_log2;   // softmax scale * log2(e)
+};
+
+// Parameters of the fp32 CUDA-core path and of the append kernels.
+struct SimtParams {
+  const void* q;
+  const void* k_cache;
+  const void* v_cache;
+  const int32_t* cache_lens;
+  const int32_t* page_table;
+  const int32_t* n_slots;
+  const int32_t* slot_len;
+  const int32_t* mask_mode;
+  const int32_t* q_row_offsets;
+  void* out;
+  int* err;
+  int B, Hq, Hkv, D;
+  int max_rows, total_rows, capacity;
+  int page_size, max_pages, n_pages;
+  float scale;
+};
+
+struct AppendParams {
+  const void* k_new;
+  const void* v_new;
+  const int32_t* accept_len;
+  void* k_cache;
+  void* v_cache;
+  int32_t* cache_lens;
+  const int32_t* page_table;
+  const int32_t* q_row_offsets;
+  int* err;
+  int B, row_bytes;  // row_bytes = Hkv * D * element size (multiple of 16)
+  int max_rows, total_rows, capacity;
+  int page_size, max_pages, n_pages;
+};
+
+// Dynamic shared memory of the tensor-core kernel.
+size_t tc_smem_bytes();
+
+cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map_k,
+                                const CUtensorMap& map_v, const TcParams& p,
+                                cudaStream_t stream);
+cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream);
+cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream);
+
+// Address of the error word on the current device (set-up once per device).
+int* device_error_word(cudaError_t* status);
+
+// Records `code` in the error word unless an earlier error is already there.
+__device__ __forceinline__ void record_error(int* err, int code) {
+  atomicCAS(err, 0, code);
+}
+
+}  // namespace zarya

@@ -1,0 +1,235 @@
+// CUDA-core kernels of the library:
+//   * slot attention in true fp32 (the fp32 storage type; tensor-core tf32
+//     would not meet fp32 accuracy), one warp per (sequence, query head, row);
+//   * KV append of accepted tokens (Sec. 5.2 step 7): 16-byte vector copies of
+//     whole token rows (Hkv * D contiguous elements) into the cache, through
+//     the page table when paged, followed by the length advance;
+//   * the per-device error word.
+#include <cuda_runtime.h>
+
+#include "internal.cuh"
+
+namespace zarya {
+
+// One error word per device that loads the library (zero = no error).
+__device__ int g_error_word = 0;
+
+int* device_error_word(cudaError_t* status) {
+  constexpr int kMaxDevices = 64;
+  static int* cache[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    if (status) *status = (e != cudaSuccess) ? e : cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  int* ptr = __atomic_load_n(&cache[dev], __ATOMIC_ACQUIRE);
+  if (ptr == nullptr) {
+    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&ptr), g_error_word);
+    if (e != cudaSuccess) {
+      if (status) *status = e;
+      return nullptr;
+    }
+    __atomic_store_n(&cache[dev], ptr, __ATOMIC_RELEASE);
+  }
+  if (status) *status = cudaSuccess;
+  return ptr;
+}
+
+namespace {
+
+// Validates sequence b of an attention call; returns its error code or 0.
+__device__ __forceinline__ int check_sequence(const SimtParams& p, int b, int* P_out, int* R_out,
+                                              int* mode_out, int* row0_out) {
+  const int P = p.cache_lens[b];
+  const int R = p.n_slots[b] * p.slot_len[b];
+  const int mode = p.mask_mode[b];
+  const int row0 = p.q_row_offsets[b];
+  const int row_end = p.q_row_offsets[b + 1];
+  *P_out = P;
+  *R_out = R;
+  *mode_out = mode;
+  *row0_out = row0;
+  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL) return ZARYA_DEVERR_MASK_MODE;
+  if (R <= 0 || R > p.max_rows || row_end - row0 != R || row0 < 0 || row_end > p.total_rows)
+    return ZARYA_DEVERR_ROWS;
+  if (P < 0 || static_cast<long long>(P) + R > p.capacity) return ZARYA_DEVERR_CAPACITY;
+  return 0;
+}
+
+// Token row index (in units of Hkv * D elements) of logical token c of
+// sequence b, or -1 when the page id is out of range.
+__device__ __forceinline__ long long token_row(const int32_t* page_table, int page_size,
+                                               int max_pages, int n_pages, int capacity, int b,
+                                               int c) {
+  if (page_size == 0) return static_cast<long long>(b) * capacity + c;
+  const int page = page_table[static_cast<long long>(b) * max_pages + c / page_size];
+  if (page < 0 || page >= n_pages) return -1;
+  return static_cast<long long>(page) * page_size + c % page_size;
+}
+
+template <int kPerLane>
+__global__ void __launch_bounds__(256)
+slot_attn_f32_kernel(const SimtParams p) {
+  constexpr int D = kPerLane * 32;
+  const int lane = threadIdx.x & 31;
+  const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long per_b = static_cast<long long>(p.Hq) * p.max_rows;
+  const int b = static_cast<int>(wid / per_b);
+  if (b >= p.B) return;
+  const int rem = static_cast<int>(wid - b * per_b);
+  const int h = rem / p.max_rows;
+  const int r = rem - h * p.max_rows;
+  int P, R, mode, row0;
+  const int code = check_sequence(p, b, &P, &R, &mode, &row0);
+  if (code != 0) {
+    if (h == 0 && r == 0 && lane == 0) record_error(p.err, code);
+    return;
+  }
+  if (r >= R) return;
+  const int g = p.Hq / p.Hkv;
+  const int j = h / g;
+  const int n_vis = (mode == ZARYA_MASK_BIDIR_BLOCK) ? P + R : P + r + 1;
+  const float* q = reinterpret_cast<const float*>(p.q) +
+                   (static_cast<long long>(row0 + r) * p.Hq + h) * D;
+  const float* kc = reinterpret_cast<const float*>(p.k_cache);
+  const float* vc = reinterpret_cast<const float*>(p.v_cache);
+  float qv[kPerLane], o[kPerLane];
+#pragma unroll
+  for (int x = 0; x < kPerLane; ++x) {
+    qv[x] = q[lane + 32 * x];
+    o[x] = 0.f;
+  }
+  float m = -INFINITY, l = 0.f;
+  for (int c = 0; c < n_vis; ++c) {
+    const long long tr =
+        token_row(p.page_table, p.page_size, p.max_pages, p.n_pages, p.capacity, b, c);
+    if (tr < 0) {
+      if (lane == 0) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+      return;
+    }
+    const long long base = (tr * p.Hkv + j) * D;
+    float dot = 0.f;
+#pragma unroll
+    for (int x = 0; x < kPerLane; ++x) dot = fmaf(qv[x], kc[base + lane + 32 * x], dot);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    const float s = dot * p.scale;
+    const float m_new = fmaxf(m, s);
+    const float corr = (m == -INFINITY) ? 0.f : expf(m - m_new);
+    const float w = expf(s - m_new);
+    l = l * corr + w;
+#pragma unroll
+    for (int x = 0; x < kPerLane; ++x) o[x] = fmaf(w, vc[base + lane + 32 * x], o[x] * corr);
+    m = m_new;
+  }
+  float* out = reinterpret_cast<float*>(p.out) + (static_cast<long long>(row0 + r) * p.Hq + h) * D;
+#pragma unroll
+  for (int x = 0; x < kPerLane; ++x) out[lane + 32 * x] = o[x] / l;
+}
+
+constexpr int kAppendRowsPerBlock = 8;
+
+// Copies rows i < accept_len[b] of the block (chunk blockIdx.x of
+// kAppendRowsPerBlock rows, sequence blockIdx.y) to cache positions P_b + i.
+__global__ void __launch_bounds__(256)
+kv_append_copy_kernel(const AppendParams p) {
+  const int b = blockIdx.y;
+  const int a = p.accept_len[b];
+  const int P = p.cache_lens[b];
+  const int row0 = p.q_row_offsets[b];
+  const int R = p.q_row_offsets[b + 1] - row0;
+  int code = 0;
+  if (R < 0 || R > p.max_rows || row0 < 0 || row0 + R > p.total_rows) code = ZARYA_DEVERR_ROWS;
+  else if (a < 0 || a > R) code = ZARYA_DEVERR_ACCEPT;
+  else if (P < 0 || static_cast<long long>(P) + a > p.capacity) code = ZARYA_DEVERR_CAPACITY;
+  if (code != 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_error(p.err, code);
+    return;
+  }
+  const int i0 = blockIdx.x * kAppendRowsPerBlock;
+  if (i0 >= a) return;
+  const int n_rows = min(kAppendRowsPerBlock, a - i0);
+  const int vec_per_row = p.row_bytes >> 4;
+  const uint4* kn = reinterpret_cast<const uint4*>(p.k_new);
+  const uint4* vn = reinterpret_cast<const uint4*>(p.v_new);
+  uint4* kc = reinterpret_cast<uint4*>(p.k_cache);
+  uint4* vc = reinterpret_cast<uint4*>(p.v_cache);
+  const int total = n_rows * vec_per_row;
+  for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
+    const int ri = idx / vec_per_row;
+    const int v = idx - ri * vec_per_row;
+    const int i = i0 + ri;
+    const int t = P + i;
+    long long tr;
+    if (p.page_size == 0) {
+      tr = static_cast<long long>(b) * p.capacity + t;
+    } else {
+      const int page = p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
+      if (page < 0 || page >= p.n_pages) {
+        record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+        continue;
+      }
+      tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+    }
+    const long long src = static_cast<long long>(row0 + i) * vec_per_row + v;
+    const long long dst = tr * vec_per_row + v;
+    kc[dst] = __ldg(kn + src);
+    vc[dst] = __ldg(vn + src);
+  }
+}
+
+// cache_lens[b] += accept_len[b] for every sequence whose copy was valid.
+__global__ void kv_append_advance_kernel(const AppendParams p) {
+  for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < p.B; b += gridDim.x * blockDim.x) {
+    const int a = p.accept_len[b];
+    const int P = p.cache_lens[b];
+    const int row0 = p.q_row_offsets[b];
+    const int R = p.q_row_offsets[b + 1] - row0;
+    if (R < 0 || R > p.max_rows || row0 < 0 || row0 + R > p.total_rows || a < 0 || a > R || P < 0 ||
+        static_cast<long long>(P) + a > p.capacity)
+      continue;
+    p.cache_lens[b] = P + a;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream) {
+  const long long warps = static_cast<long long>(p.B) * p.Hq * p.max_rows;
+  const long long threads = warps * 32;
+  const int block = 256;
+  const long long grid = (threads + block - 1) / block;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  switch (p.D / 32) {
+    case 1: slot_attn_f32_kernel<1><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 2: slot_attn_f32_kernel<2><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 3: slot_attn_f32_kernel<3><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 4: slot_attn_f32_kernel<4><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 5: slot_attn_f32_kernel<5><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 6: slot_attn_f32_kernel<6><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 7: slot_attn_f32_kernel<7><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 8: slot_attn_f32_kernel<8><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream) {
+  const int chunks = (p.max_rows + kAppendRowsPerBlock - 1) / kAppendRowsPerBlock;
+  if (chunks > 0) {
+    dim3 grid(chunks, p.B);
+    kv_append_copy_kernel<<<grid, 256, 0, stream>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  if (commit) {
+    const int block = 128;
+    const int grid = (p.B + block - 1) / block;
+    kv_append_advance_kernel<<<grid, block, 0, stream>>>(p);
+    return cudaGetLastError();
+  }
+  return cudaSuccess;
+}
+
+}  // namespace zarya

@@ -1,0 +1,137 @@
+"""CPU checks of the C ABI: the library loads, exports every function that
+include/zarya.h declares, and rejects invalid calls on the host (before any
+CUDA call, so no GPU is needed)."""
+import ctypes
+
+import pytest
+
+from paper_2609_19868_gb300 import _binding as zb
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_19868_gb300 import build
+
+    build.build()
+    return zb.load()
+
+
+def _desc(**kw):
+    d = zb.AttnDesc()
+    base = dict(batch=2, n_q_heads=16, n_kv_heads=8, head_dim=128, dtype=zb.BF16, page_size=0,
+                cache_capacity=256, n_pages=0, max_rows=32, total_rows=64, max_kv_len=0,
+                kv_splits=0, scale=0.0, q_row_offsets=0x100000)
+    base.update(kw)
+    for k, v in base.items():
+        setattr(d, k, v)
+    return d
+
+
+FAKE = 0x7F0000000000  # never dereferenced: validation fails before any access
+
+
+def _attn(lib, d, q=FAKE, k=FAKE, v=FAKE, out=FAKE, page_table=None, ws=None, ws_bytes=0):
+    vp = ctypes.c_void_p
+    return lib.zarya_slot_attn(vp(q), vp(k), vp(v), vp(FAKE), vp(page_table), vp(FAKE), vp(FAKE),
+                               vp(FAKE), vp(out), vp(ws), ws_bytes,
+                               None if d is None else ctypes.byref(d), None)
+
+
+def test_exports_every_declared_function(lib):
+    names = zb.header_functions()
+    assert {"zarya_slot_attn", "zarya_kv_append", "zarya_slot_attn_workspace_size",
+            "zarya_check_device_error", "zarya_status_string", "zarya_version"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_and_version(lib):
+    assert zb.status_string(0) == "ok"
+    assert zb.status_string(2) == "unsupported configuration"
+    assert zb.status_string(99) == "unknown status"
+    assert zb.version() >= 100
+
+
+def test_desc_struct_layout_matches_c():
+    # 12 int32 + float, then a pointer aligned to 8
+    assert ctypes.sizeof(zb.AttnDesc) == 64
+    assert zb.AttnDesc.q_row_offsets.offset == 56
+
+
+@pytest.mark.parametrize("bad,status", [
+    (dict(batch=0), 1),
+    (dict(n_q_heads=12, n_kv_heads=8), 1),
+    (dict(dtype=7), 1),
+    (dict(max_rows=0), 1),
+    (dict(total_rows=0), 1),
+    (dict(cache_capacity=0), 1),
+    (dict(page_size=16, cache_capacity=250, n_pages=10), 1),
+    (dict(page_size=16, cache_capacity=256, n_pages=0), 1),
+    (dict(scale=-1.0), 1),
+    (dict(scale=float("nan")), 1),
+    (dict(q_row_offsets=0), 1),
+    (dict(kv_splits=-2), 1),
+    (dict(head_dim=64), 2),                       # bf16 tensor-core path is D = 128
+    (dict(n_q_heads=24, n_kv_heads=8), 2),        # group of 3 does not divide 128 rows
+    (dict(page_size=8, cache_capacity=256, n_pages=40), 2),
+    (dict(dtype=zb.FP32, head_dim=48), 2),
+])
+def test_attention_rejects_invalid_descriptors(lib, bad, status):
+    assert _attn(lib, _desc(**bad)) == status
+
+
+def test_attention_rejects_null_and_misaligned_pointers(lib):
+    assert _attn(lib, None) == 1
+    assert _attn(lib, _desc(), q=None) == 1
+    assert _attn(lib, _desc(), out=FAKE + 8) == 1
+    assert _attn(lib, _desc(), k=FAKE + 2) == 1
+    # page table given for a contiguous cache, or missing for a paged one
+    assert _attn(lib, _desc(), page_table=FAKE) == 1
+    assert _attn(lib, _desc(page_size=16, n_pages=64), page_table=None) == 1
+
+
+def test_workspace_size_is_zero_for_invalid_or_fp32(lib):
+    assert lib.zarya_slot_attn_workspace_size(None) == 0
+    assert lib.zarya_slot_attn_workspace_size(ctypes.byref(_desc(batch=0))) == 0
+    assert lib.zarya_slot_attn_workspace_size(ctypes.byref(_desc(dtype=zb.FP32, head_dim=64))) == 0
+
+
+def test_workspace_size_for_forced_splits(lib):
+    # 2 sequences x 8 KV heads x 1 M-tile, 3 splits: partial O + lse + counters
+    d = _desc(kv_splits=3, cache_capacity=512)
+    n = 2 * 8 * 1 * 3 * 128
+    expect = n * 128 * 4
+    expect = (expect + 255) // 256 * 256 + n * 4
+    expect = (expect + 255) // 256 * 256 + 16 * 4
+    expect = (expect + 255) // 256 * 256
+    assert lib.zarya_slot_attn_workspace_size(ctypes.byref(d)) == expect
+    assert lib.zarya_slot_attn_workspace_size(ctypes.byref(_desc(kv_splits=1))) == 0
+
+
+def test_attention_requires_large_enough_workspace(lib):
+    d = _desc(kv_splits=2)
+    need = lib.zarya_slot_attn_workspace_size(ctypes.byref(d))
+    assert need > 0
+    # validation of the workspace happens after device selection, which needs
+    # a GPU; on a CPU-only host the call must still fail cleanly (no crash)
+    st = _attn(lib, d, ws=None, ws_bytes=0)
+    assert st in (1, 3)
+
+
+def test_append_rejects_invalid_calls(lib):
+    vp = ctypes.c_void_p
+    d = _desc()
+
+    def app(flags=1, k_new=FAKE, desc=d, page_table=None, accept=FAKE):
+        return lib.zarya_kv_append(vp(k_new), vp(FAKE), vp(accept), vp(FAKE), vp(FAKE), vp(FAKE),
+                                   vp(page_table), flags,
+                                   None if desc is None else ctypes.byref(desc), None)
+
+    assert app(flags=2) == 1
+    assert app(flags=-1) == 1
+    assert app(desc=None) == 1
+    assert app(k_new=None) == 1
+    assert app(accept=None) == 1
+    assert app(k_new=FAKE + 4) == 1
+    assert app(page_table=FAKE) == 1
+    assert app(desc=_desc(n_kv_heads=1, n_q_heads=1, head_dim=4)) == 2  # row not 16-byte multiple

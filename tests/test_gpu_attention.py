@@ -1,0 +1,152 @@
+"""GPU parity of zarya_slot_attn against the fp64 CPU oracle.
+
+Every test calls the CUDA library through the C ABI (the ctypes binding) on
+seeded synthetic inputs of the five workloads; the oracle sees the same
+bytes. Reduced workloads are compared element by element on every output;
+full-size workloads, in the launch configuration the benchmark uses, on
+sampled rows the oracle computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_19868_gb300 import workloads as wl
+from _helpers import (gather_rows, oracle_full, oracle_rows, oracle_staged, sample_rows,
+                      tolerance_ok)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def zs():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_19868_gb300 import build, session
+    from paper_2609_19868_gb300 import _binding as zb
+
+    build.build()
+    zb.load()
+    zb.check_device_error()
+    return session, zb
+
+
+def _cases():
+    out = []
+    for name in wl.ORDER:
+        spec = wl.SPECS[name]
+        if spec["mode"][0] == "both":
+            out += [(name, 0), (name, 1)]
+        else:
+            out.append((name, None))
+    return out
+
+
+def _run(zs, w, mode=None, kv_splits=0):
+    session, zb = zs
+    db = session.upload(w, "cuda", kv_splits=kv_splits, mask_mode=mode)
+    db.stage()
+    db.attend()
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    return db
+
+
+@pytest.mark.parametrize("name,mode", _cases())
+def test_reduced_workload_matches_oracle_everywhere(zs, oracle_mod, name, mode):
+    w = wl.make(name, small=True)
+    db = _run(zs, w, mode)
+    kc, vc = oracle_staged(oracle_mod, w)
+    ref = oracle_full(oracle_mod, w, kc, vc, mode)
+    got = db.out
+    assert not torch.isnan(got).any()
+    ok, err, scale = tolerance_ok(got, ref, w.dtype)
+    assert ok, f"{name} mode={mode}: max|err|={err:.3e} max|ref|={scale:.3f}"
+
+
+@pytest.mark.parametrize("name,mode", [("decode_small", None), ("long_ctx", 0), ("long_ctx", 1),
+                                       ("ragged_mid", None)])
+@pytest.mark.parametrize("splits", [1, 2, 3, 7])
+def test_split_kv_merge_matches_oracle(zs, oracle_mod, name, mode, splits):
+    """Forcing the key range to be split n ways (partials merged in-kernel by
+    the last CTA to arrive) still matches the oracle."""
+    w = wl.make(name, small=True)
+    db = _run(zs, w, mode, kv_splits=splits)
+    kc, vc = oracle_staged(oracle_mod, w)
+    ref = oracle_full(oracle_mod, w, kc, vc, mode)
+    ok, err, scale = tolerance_ok(db.out, ref, w.dtype)
+    assert ok, f"{name} splits={splits}: max|err|={err:.3e}"
+
+
+def test_workspace_counters_return_to_zero(zs):
+    """The split merge leaves its arrival counters at zero, so a workspace
+    can be reused: two calls in a row give identical results."""
+    w = wl.make("decode_small", small=True)
+    session, zb = zs
+    db = session.upload(w, "cuda", kv_splits=3)
+    db.stage()
+    db.attend()
+    first = db.out.clone()
+    db.out.zero_()
+    db.attend()
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    assert torch.equal(first, db.out)
+    # the counters are the last units*4 bytes (rounded) of the workspace
+    assert db.workspace is not None
+
+
+def test_repeat_runs_are_bitwise_deterministic(zs):
+    w = wl.make("serving_mix", small=True)
+    a = _run(zs, w).out.clone()
+    b = _run(zs, w).out.clone()
+    assert torch.equal(a, b)
+
+
+def test_paged_cache_equals_contiguous_bitwise(zs):
+    """The same logical keys behind a random page table give bit-identical
+    outputs (same key tiles, same order)."""
+    session, zb = zs
+    wc = wl.make("ragged_mid", small=True)
+    rng = np.random.default_rng(5)
+    ps = 16
+    P = wc.cache_lens.astype(np.int64)
+    R = wc.R
+    npg = (P + R + ps - 1) // ps
+    n_pages = int(npg.sum()) + 3
+    perm = rng.permutation(n_pages)
+    pt = np.full((wc.B, int(npg.max())), -1, dtype=np.int32)
+    kp = torch.full((n_pages, ps, wc.Hkv, wc.D), float("nan"), dtype=torch.bfloat16)
+    vp = torch.full_like(kp, float("nan"))
+    start = 0
+    for b in range(wc.B):
+        pt[b, :npg[b]] = perm[start:start + npg[b]]
+        start += int(npg[b])
+        for lp in range(int(npg[b])):
+            lo = lp * ps
+            hi = min(lo + ps, int(P[b]))
+            if hi > lo:
+                kp[pt[b, lp], :hi - lo] = wc.k_cache[b, lo:hi]
+                vp[pt[b, lp], :hi - lo] = wc.v_cache[b, lo:hi]
+    from dataclasses import replace
+    wp = replace(wc, page_size=ps, capacity=int(npg.max()) * ps, n_pages=n_pages, page_table=pt,
+                 k_cache=kp, v_cache=vp)
+    oc = _run(zs, wc, kv_splits=1).out
+    op = _run(zs, wp, kv_splits=1).out
+    assert torch.equal(oc, op)
+
+
+@pytest.mark.parametrize("name,mode", _cases())
+def test_full_size_sampled_rows_match_oracle(zs, oracle_mod, name, mode):
+    """Full-size workloads in the benchmark's launch configuration (automatic
+    split plan): sampled (sequence, head, row) outputs against the oracle."""
+    w = wl.make(name)
+    db = _run(zs, w, mode)
+    out = db.out
+    assert not torch.isnan(out).any()
+    del db
+    kc, vc = oracle_staged(oracle_mod, w)
+    sel = sample_rows(w, 192, seed=7)
+    ref = oracle_rows(oracle_mod, w, kc, vc, sel, mode)
+    got = gather_rows(out, w, sel)
+    ok, err, scale = tolerance_ok(got, ref, w.dtype)
+    assert ok, f"{name} mode={mode}: max|err|={err:.3e} max|ref|={scale:.3f}"
