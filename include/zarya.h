@@ -134,6 +134,35 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
                              zarya_stream_t stream);
 
 /*
+ * zarya_slot_attn without a workspace argument, for callers that cannot
+ * allocate device memory at the point where they run attention: a serving
+ * engine that has already given all of HBM to its own cache pool, a host
+ * application whose plug-ins may not allocate device memory, or a decode loop
+ * that cannot afford cudaMalloc / cudaFree (both can synchronise the device).
+ * The paper has no counterpart; this is a deployment convenience.
+ *
+ * Same arguments, results and errors as zarya_slot_attn, minus workspace.
+ * The split-KV scratch is a 16 MiB array inside the library, reserved on
+ * every GPU that loads it until the process exits; this call allocates
+ * nothing. A descriptor whose split plan needs more than 16 MiB
+ * (zarya_slot_attn_workspace_size(desc) > 16 MiB) is rejected with
+ * ZARYA_ERR_UNSUPPORTED and nothing is launched; set desc->kv_splits = 1
+ * (no scratch needed) or use zarya_slot_attn with a workspace.
+ * The first call on each device looks up the scratch address on that device
+ * (a one-time set-up step); make that first call before any stream capture.
+ * Every call on a device shares the one scratch array, which keeps what the
+ * last call left: each call zeroes the part that must start at zero (the
+ * split arrival counters) on `stream` before its kernel runs, so calls in
+ * order on one stream are safe, but calls that overlap on the GPU (different
+ * streams, or different threads) race on the scratch and give wrong results.
+ */
+zarya_status zarya_slot_attn_noalloc(const void* q, const void* k_cache, const void* v_cache,
+                                     const int32_t* cache_lens, const int32_t* page_table,
+                                     const int32_t* n_slots, const int32_t* slot_len,
+                                     const int32_t* mask_mode, void* out,
+                                     const zarya_attn_desc* desc, zarya_stream_t stream);
+
+/*
  * KV-cache update with accepted tokens (Sec. 5.2 step 7): for every sequence
  * b and i < accept_len[b], row q_row_offsets[b] + i of k_new / v_new
  * ([total_rows, Hkv, D], the block rows in reordered order, accepted tokens

@@ -68,6 +68,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_slot_attn_workspace_size.restype = sz
     lib.zarya_slot_attn.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, dp, vp]
     lib.zarya_slot_attn.restype = ctypes.c_int
+    lib.zarya_slot_attn_noalloc.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, vp]
+    lib.zarya_slot_attn_noalloc.restype = ctypes.c_int
     lib.zarya_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, dp, vp]
     lib.zarya_kv_append.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
@@ -153,6 +155,28 @@ def slot_attn(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len, ma
                                 ctypes.byref(desc), _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_slot_attn")
+
+
+def slot_attn_noalloc(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len,
+                      mask_mode, out, desc: AttnDesc, stream=None) -> None:
+    """``zarya_slot_attn_noalloc``: slot attention for callers that cannot
+    allocate device memory when they run it. Its split-KV scratch is a fixed
+    16 MiB array inside the library (one per GPU), so no workspace is passed
+    and nothing is allocated; plans that need more scratch are rejected.
+    Calls that overlap on the GPU share that array and must not be issued."""
+    for name, t in (("q", q), ("k_cache", k_cache), ("v_cache", v_cache), ("out", out)):
+        _check_cuda(name, t)
+    for name, t in (("cache_lens", cache_lens), ("n_slots", n_slots), ("slot_len", slot_len),
+                    ("mask_mode", mask_mode)):
+        _check_cuda(name, t, torch.int32)
+    if page_table is not None:
+        _check_cuda("page_table", page_table, torch.int32)
+    st = load().zarya_slot_attn_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_lens),
+                                        _ptr(page_table), _ptr(n_slots), _ptr(slot_len),
+                                        _ptr(mask_mode), _ptr(out), ctypes.byref(desc),
+                                        _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_slot_attn_noalloc")
 
 
 def kv_append(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, page_table,
