@@ -187,6 +187,14 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
  */
 zarya_status zarya_check_device_error(zarya_stream_t stream, int32_t* code);
 
+/*
+ * Message about the last CUDA runtime/driver failure behind a ZARYA_ERR_CUDA
+ * returned on the calling thread ("what failed: CUDA's error string (code)");
+ * empty if there was none. Owned by the library; valid until the next call
+ * on the same thread.
+ */
+const char* zarya_last_error(void);
+
 /* Static, human-readable name of a status. */
 const char* zarya_status_string(zarya_status status);
 

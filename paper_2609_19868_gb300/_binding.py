@@ -27,7 +27,10 @@ DEVERR_NAMES = {0: "none", 1: "page id", 2: "rows", 3: "capacity", 4: "accept le
 
 class ZaryaError(RuntimeError):
     def __init__(self, status: int, what: str):
-        super().__init__(f"{what}: {status_string(status)} (status {status})")
+        msg = f"{what}: {status_string(status)} (status {status})"
+        if status == ERR_CUDA:
+            msg += f" [{last_error()}]"
+        super().__init__(msg)
         self.status = status
 
 
@@ -74,6 +77,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_kv_append.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
     lib.zarya_check_device_error.restype = ctypes.c_int
+    lib.zarya_last_error.argtypes = []
+    lib.zarya_last_error.restype = ctypes.c_char_p
     lib.zarya_status_string.argtypes = [ctypes.c_int]
     lib.zarya_status_string.restype = ctypes.c_char_p
     lib.zarya_version.argtypes = []
@@ -91,6 +96,11 @@ def header_functions() -> list:
 
 def status_string(status: int) -> str:
     return load().zarya_status_string(int(status)).decode()
+
+
+def last_error() -> str:
+    """The library's message about the last CUDA failure on this thread."""
+    return load().zarya_last_error().decode()
 
 
 def version() -> int:

@@ -7,6 +7,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
 
 #include "internal.cuh"
 
@@ -29,28 +30,6 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
-// Makes the device that owns `stream` (or, for the legacy default stream, the
-// device that owns `ptr`) current for this thread.
-cudaError_t select_device(cudaStream_t stream, const void* ptr) {
-  int want = -1;
-  if (stream != nullptr) {
-    cudaError_t e = cudaStreamGetDevice(stream, &want);
-    if (e != cudaSuccess) return e;
-  } else {
-    cudaPointerAttributes attr{};
-    cudaError_t e = cudaPointerGetAttributes(&attr, ptr);
-    if (e != cudaSuccess) return e;
-    if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
-      return cudaErrorInvalidValue;
-    want = attr.device;
-  }
-  int cur = -1;
-  cudaError_t e = cudaGetDevice(&cur);
-  if (e != cudaSuccess) return e;
-  if (cur != want) return cudaSetDevice(want);
-  return cudaSuccess;
-}
 
 int sm_count() {
   constexpr int kMaxDevices = 64;
@@ -104,6 +83,8 @@ zarya_status check_attn_support(const zarya_attn_desc* d) {
   return ZARYA_OK;
 }
 
+constexpr int kMaxClusterSplits = 8;  // portable cluster size
+
 struct Plan {
   int g, m_tiles, splits;
   long long units;
@@ -128,7 +109,7 @@ Plan plan_tc(const zarya_attn_desc* d, int sms) {
     splits = d->kv_splits < tiles ? d->kv_splits : tiles;
   } else if (p.units < sms) {
     double best = 1e30;
-    for (int s = 1; s <= tiles && s <= 32; ++s) {
+    for (int s = 1; s <= tiles && s <= kMaxClusterSplits; ++s) {
       const long long waves = (p.units * s + sms - 1) / sms;
       const double cost = static_cast<double>(waves) * ((tiles + s - 1) / s + 2.0) +
                           (s > 1 ? 1.0 : 0.0);
@@ -140,7 +121,9 @@ Plan plan_tc(const zarya_attn_desc* d, int sms) {
   }
   if (splits < 1) splits = 1;
   p.splits = splits;
-  if (splits > 1) {
+  // Up to kMaxClusterSplits splits merge through distributed shared memory
+  // inside a thread-block cluster; more splits merge through the workspace.
+  if (splits > kMaxClusterSplits) {
     const size_t n = static_cast<size_t>(p.units) * splits * kBlockM;
     const size_t bytes_o = n * kHeadDim * sizeof(float);
     p.off_lse = align256(bytes_o);
@@ -161,6 +144,51 @@ CUresult encode(CUtensorMap* map, void* base, cuuint32_t rank, const cuuint64_t*
 }
 
 }  // namespace
+
+// Makes the device that owns `stream` current for this thread. The stream is
+// asked directly unless it is capturing into a CUDA graph (where that query is
+// not permitted) or is the legacy default stream; then the device that owns
+// `ptr` (a device buffer of the call) is used.
+cudaError_t select_device(cudaStream_t stream, const void* ptr) {
+  int want = -1;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (stream != nullptr) {
+    cudaError_t e = cudaStreamIsCapturing(stream, &cs);
+    if (e != cudaSuccess) return e;
+  }
+  if (stream != nullptr && cs == cudaStreamCaptureStatusNone) {
+    cudaError_t e = cudaStreamGetDevice(stream, &want);
+    if (e != cudaSuccess) return e;
+  } else {
+    cudaPointerAttributes attr{};
+    cudaError_t e = cudaPointerGetAttributes(&attr, ptr);
+    if (e != cudaSuccess) return e;
+    if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
+      return cudaErrorInvalidValue;
+    want = attr.device;
+  }
+  int cur = -1;
+  cudaError_t e = cudaGetDevice(&cur);
+  if (e != cudaSuccess) return e;
+  if (cur != want) return cudaSetDevice(want);
+  return cudaSuccess;
+}
+
+static thread_local char g_last_error[256] = "";
+
+zarya_status cuda_fail(const char* what, cudaError_t e) {
+  std::snprintf(g_last_error, sizeof g_last_error, "%s: %s (%d)", what, cudaGetErrorString(e),
+                static_cast<int>(e));
+  return ZARYA_ERR_CUDA;
+}
+
+size_t workspace_counter_bytes(const zarya_attn_desc* desc) {
+  if (check_desc(desc) != ZARYA_OK || check_attn_support(desc) != ZARYA_OK) return 0;
+  if (desc->dtype != ZARYA_BF16) return 0;
+  const Plan plan = plan_tc(desc, sm_count());
+  return plan.bytes > 0 ? plan.bytes - plan.off_cnt : 0;
+}
+
 }  // namespace zarya
 
 using namespace zarya;
@@ -189,10 +217,10 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
   if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
     return ZARYA_ERR_INVALID_ARG;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  if (select_device(stream, q) != cudaSuccess) return ZARYA_ERR_CUDA;
-  cudaError_t ce = cudaSuccess;
+  cudaError_t ce = select_device(stream, q);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
   int* err = device_error_word(&ce);
-  if (err == nullptr) return ZARYA_ERR_CUDA;
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
   const float scale =
       desc->scale > 0.f ? desc->scale : 1.0f / std::sqrt(static_cast<float>(desc->head_dim));
   const int max_pages = desc->page_size > 0 ? desc->cache_capacity / desc->page_size : 0;
@@ -221,7 +249,8 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
     p.max_pages = max_pages;
     p.n_pages = desc->n_pages;
     p.scale = scale;
-    return launch_slot_attn_f32(p, stream) == cudaSuccess ? ZARYA_OK : ZARYA_ERR_CUDA;
+    ce = launch_slot_attn_f32(p, stream);
+    return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching slot_attn_f32_kernel", ce);
   }
 
   const Plan plan = plan_tc(desc, sm_count());
@@ -244,7 +273,7 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
     const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(g),
                                static_cast<cuuint32_t>(kBlockM / g)};
     if (encode(&map_q, const_cast<void*>(q), 3, dims, strides, box) != CUDA_SUCCESS)
-      return ZARYA_ERR_CUDA;
+      return cuda_fail("encoding the Q tensor map", cudaErrorInvalidValue);
   }
   {
     cuuint64_t dims[4], strides[3];
@@ -269,7 +298,7 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
     }
     if (encode(&map_k, const_cast<void*>(k_cache), 4, dims, strides, box) != CUDA_SUCCESS ||
         encode(&map_v, const_cast<void*>(v_cache), 4, dims, strides, box) != CUDA_SUCCESS)
-      return ZARYA_ERR_CUDA;
+      return cuda_fail("encoding the K/V tensor maps", cudaErrorInvalidValue);
   }
 
   TcParams p{};
@@ -299,9 +328,10 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
   p.n_pages = desc->n_pages;
   p.m_tiles = plan.m_tiles;
   p.splits = plan.splits;
+  p.cluster = (plan.splits > 1 && plan.splits <= kMaxClusterSplits) ? 1 : 0;
   p.scale_log2 = scale * 1.4426950408889634f;
-  return launch_slot_attn_tc(map_q, map_k, map_v, p, stream) == cudaSuccess ? ZARYA_OK
-                                                                           : ZARYA_ERR_CUDA;
+  ce = launch_slot_attn_tc(map_q, map_k, map_v, p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching slot_attn_tc_kernel", ce);
 }
 
 zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
@@ -317,10 +347,10 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
     return ZARYA_ERR_INVALID_ARG;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  if (select_device(stream, k_new) != cudaSuccess) return ZARYA_ERR_CUDA;
-  cudaError_t ce = cudaSuccess;
+  cudaError_t ce = select_device(stream, k_new);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
   int* err = device_error_word(&ce);
-  if (err == nullptr) return ZARYA_ERR_CUDA;
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
   const int eb = desc->dtype == ZARYA_BF16 ? 2 : 4;
   AppendParams p{};
   p.k_new = k_new;
@@ -341,32 +371,39 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
   p.max_pages = desc->page_size > 0 ? desc->cache_capacity / desc->page_size : 0;
   p.n_pages = desc->n_pages;
   if (desc->batch > 65535) return ZARYA_ERR_UNSUPPORTED;
-  return launch_kv_append(p, flags == ZARYA_APPEND_COMMIT, stream) == cudaSuccess
-             ? ZARYA_OK
-             : ZARYA_ERR_CUDA;
+  ce = launch_kv_append(p, flags == ZARYA_APPEND_COMMIT, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the append kernels", ce);
 }
 
 zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {
   if (code) *code = 0;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce;
   if (stream != nullptr) {
     int dev = -1, cur = -1;
-    if (cudaStreamGetDevice(stream, &dev) != cudaSuccess) return ZARYA_ERR_CUDA;
-    if (cudaGetDevice(&cur) != cudaSuccess) return ZARYA_ERR_CUDA;
-    if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return ZARYA_ERR_CUDA;
+    if ((ce = cudaStreamGetDevice(stream, &dev)) != cudaSuccess)
+      return cuda_fail("cudaStreamGetDevice", ce);
+    if ((ce = cudaGetDevice(&cur)) != cudaSuccess) return cuda_fail("cudaGetDevice", ce);
+    if (cur != dev && (ce = cudaSetDevice(dev)) != cudaSuccess)
+      return cuda_fail("cudaSetDevice", ce);
   }
-  cudaError_t ce = cudaSuccess;
   int* err = device_error_word(&ce);
-  if (err == nullptr) return ZARYA_ERR_CUDA;
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
   int host = 0;
-  if (cudaStreamSynchronize(stream) != cudaSuccess) return ZARYA_ERR_CUDA;
-  if (cudaMemcpyAsync(&host, err, sizeof(int), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
-    return ZARYA_ERR_CUDA;
-  if (cudaMemsetAsync(err, 0, sizeof(int), stream) != cudaSuccess) return ZARYA_ERR_CUDA;
-  if (cudaStreamSynchronize(stream) != cudaSuccess) return ZARYA_ERR_CUDA;
+  if ((ce = cudaStreamSynchronize(stream)) != cudaSuccess)
+    return cuda_fail("cudaStreamSynchronize", ce);
+  if ((ce = cudaMemcpyAsync(&host, err, sizeof(int), cudaMemcpyDeviceToHost, stream)) !=
+      cudaSuccess)
+    return cuda_fail("reading the device error word", ce);
+  if ((ce = cudaMemsetAsync(err, 0, sizeof(int), stream)) != cudaSuccess)
+    return cuda_fail("clearing the device error word", ce);
+  if ((ce = cudaStreamSynchronize(stream)) != cudaSuccess)
+    return cuda_fail("cudaStreamSynchronize", ce);
   if (code) *code = host;
   return host == 0 ? ZARYA_OK : ZARYA_ERR_DEVICE_FAULT;
 }
+
+const char* zarya_last_error(void) { return g_last_error; }
 
 const char* zarya_status_string(zarya_status status) {
   switch (status) {

@@ -27,12 +27,13 @@ struct TcParams {
   void* out;          // bf16 [total_rows, Hq, D]
   float* ws_o;        // [units, splits, kBlockM, D] fp32 partial outputs (normalised)
   float* ws_lse;      // [units, splits, kBlockM] log2-sum-exp of each partial
-  int32_t* ws_count;  // [units] arrival counters (zero between calls)
+  int32_t* ws_count;  // [units] arrival counters of the workspace merge (zero between calls)
   int* err;           // device error word
   int B, Hq, Hkv, g;
   int max_rows, total_rows, capacity;
   int page_size, max_pages, n_pages;
   int m_tiles, splits;
+  int cluster;        // 1: the splits of a tile form a cluster and merge through DSMEM
   float scale_log2;   // softmax scale * log2(e)
 };
 
@@ -78,6 +79,35 @@ cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map
                                 cudaStream_t stream);
 cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream);
 cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream);
+
+// Bytes at the end of the attention workspace that hold the split counters
+// (which must be zero before a call); 0 when the plan needs no workspace.
+size_t workspace_counter_bytes(const zarya_attn_desc* desc);
+
+// Launch configuration with programmatic stream serialisation enabled, so a
+// kernel's set-up can overlap the tail of the kernel before it.
+struct PdlLaunch {
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  PdlLaunch(dim3 grid, dim3 block, size_t smem, cudaStream_t stream) : cfg{}, attr{} {
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+};
+
+// Makes the device that owns `stream` (or, while it captures a graph or for
+// the legacy default stream, the device that owns `ptr`) current.
+cudaError_t select_device(cudaStream_t stream, const void* ptr);
+
+// Records "what: <CUDA error string>" as this thread's last error message
+// (zarya_last_error) and returns ZARYA_ERR_CUDA.
+zarya_status cuda_fail(const char* what, cudaError_t e);
 
 // Address of the error word on the current device (set-up once per device).
 int* device_error_word(cudaError_t* status);

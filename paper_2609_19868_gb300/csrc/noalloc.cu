@@ -61,38 +61,22 @@ zarya_status zarya_slot_attn_noalloc(const void* q, const void* k_cache, const v
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   // Make the stream's device current: the scratch address and the split plan
   // (which depends on the SM count) are per device.
-  int want = -1;
-  if (stream != nullptr) {
-    if (cudaStreamGetDevice(stream, &want) != cudaSuccess) return ZARYA_ERR_CUDA;
-  } else {
-    cudaPointerAttributes attr{};
-    if (cudaPointerGetAttributes(&attr, q) != cudaSuccess) return ZARYA_ERR_CUDA;
-    if (attr.type != cudaMemoryTypeDevice && attr.type != cudaMemoryTypeManaged)
-      return ZARYA_ERR_INVALID_ARG;
-    want = attr.device;
-  }
-  int cur = -1;
-  if (cudaGetDevice(&cur) != cudaSuccess) return ZARYA_ERR_CUDA;
-  if (cur != want && cudaSetDevice(want) != cudaSuccess) return ZARYA_ERR_CUDA;
+  cudaError_t ce = zarya::select_device(stream, q);
+  if (ce != cudaSuccess) return zarya::cuda_fail("selecting the stream's device", ce);
 
   const size_t need = zarya_slot_attn_workspace_size(desc);
   if (need > zarya::kScratchBytes) return ZARYA_ERR_UNSUPPORTED;
   void* scratch = nullptr;
   if (need > 0) {
-    cudaError_t ce = cudaSuccess;
     scratch = zarya::scratch_address(&ce);
-    if (scratch == nullptr) return ZARYA_ERR_CUDA;
-    // The per-tile arrival counters sit at the end of the workspace layout
-    // and must start at zero; the array keeps whatever the last call left.
-    const int g = desc->n_q_heads / desc->n_kv_heads;
-    const long long m_tiles =
-        (static_cast<long long>(desc->max_rows) * g + zarya::kBlockM - 1) / zarya::kBlockM;
-    const long long units = static_cast<long long>(desc->batch) * desc->n_kv_heads * m_tiles;
-    const size_t cnt_bytes = (static_cast<size_t>(units) * sizeof(int32_t) + 255) & ~size_t(255);
-    if (cnt_bytes > need) return ZARYA_ERR_CUDA;
-    if (cudaMemsetAsync(static_cast<unsigned char*>(scratch) + (need - cnt_bytes), 0, cnt_bytes,
-                        stream) != cudaSuccess)
-      return ZARYA_ERR_CUDA;
+    if (scratch == nullptr) return zarya::cuda_fail("looking up the scratch address", ce);
+    // The split counters sit at the end of the workspace layout and must
+    // start at zero; the array keeps whatever the last call left.
+    const size_t cnt_bytes = zarya::workspace_counter_bytes(desc);
+    if (cnt_bytes == 0 || cnt_bytes > need) return ZARYA_ERR_CUDA;
+    ce = cudaMemsetAsync(static_cast<unsigned char*>(scratch) + (need - cnt_bytes), 0, cnt_bytes,
+                         stream);
+    if (ce != cudaSuccess) return zarya::cuda_fail("clearing the split counters", ce);
   }
   return zarya_slot_attn(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len,
                          mask_mode, out, scratch, need > 0 ? zarya::kScratchBytes : 0, desc,

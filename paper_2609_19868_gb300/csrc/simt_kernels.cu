@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace zarya {
 
@@ -71,6 +72,8 @@ __device__ __forceinline__ long long token_row(const int32_t* page_table, int pa
 template <int kPerLane>
 __global__ void __launch_bounds__(256)
 slot_attn_f32_kernel(const SimtParams p) {
+  grid_dependency_wait();
+  grid_launch_dependents();
   constexpr int D = kPerLane * 32;
   const int lane = threadIdx.x & 31;
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -134,6 +137,8 @@ constexpr int kAppendRowsPerBlock = 8;
 // kAppendRowsPerBlock rows, sequence blockIdx.y) to cache positions P_b + i.
 __global__ void __launch_bounds__(256)
 kv_append_copy_kernel(const AppendParams p) {
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int b = blockIdx.y;
   const int a = p.accept_len[b];
   const int P = p.cache_lens[b];
@@ -181,6 +186,8 @@ kv_append_copy_kernel(const AppendParams p) {
 
 // cache_lens[b] += accept_len[b] for every sequence whose copy was valid.
 __global__ void kv_append_advance_kernel(const AppendParams p) {
+  grid_dependency_wait();
+  grid_launch_dependents();
   for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < p.B; b += gridDim.x * blockDim.x) {
     const int a = p.accept_len[b];
     const int P = p.cache_lens[b];
@@ -201,33 +208,31 @@ cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream) {
   const int block = 256;
   const long long grid = (threads + block - 1) / block;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+  PdlLaunch l(dim3(static_cast<unsigned>(grid)), dim3(block), 0, stream);
   switch (p.D / 32) {
-    case 1: slot_attn_f32_kernel<1><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 2: slot_attn_f32_kernel<2><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 3: slot_attn_f32_kernel<3><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 4: slot_attn_f32_kernel<4><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 5: slot_attn_f32_kernel<5><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 6: slot_attn_f32_kernel<6><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 7: slot_attn_f32_kernel<7><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
-    case 8: slot_attn_f32_kernel<8><<<static_cast<unsigned>(grid), block, 0, stream>>>(p); break;
+    case 1: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<1>, p);
+    case 2: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<2>, p);
+    case 3: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<3>, p);
+    case 4: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<4>, p);
+    case 5: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<5>, p);
+    case 6: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<6>, p);
+    case 7: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<7>, p);
+    case 8: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<8>, p);
     default: return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream) {
   const int chunks = (p.max_rows + kAppendRowsPerBlock - 1) / kAppendRowsPerBlock;
   if (chunks > 0) {
-    dim3 grid(chunks, p.B);
-    kv_append_copy_kernel<<<grid, 256, 0, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
+    PdlLaunch l(dim3(chunks, p.B), dim3(256), 0, stream);
+    cudaError_t e = cudaLaunchKernelEx(&l.cfg, kv_append_copy_kernel, p);
     if (e != cudaSuccess) return e;
   }
   if (commit) {
     const int block = 128;
-    const int grid = (p.B + block - 1) / block;
-    kv_append_advance_kernel<<<grid, block, 0, stream>>>(p);
-    return cudaGetLastError();
+    PdlLaunch l(dim3((p.B + block - 1) / block), dim3(block), 0, stream);
+    return cudaLaunchKernelEx(&l.cfg, kv_append_advance_kernel, p);
   }
   return cudaSuccess;
 }

@@ -10,19 +10,25 @@
 //     128/g block rows (packed row m -> block row r0 + m/g, head j*g + m%g),
 //     loaded by one 3-D TMA box per 64-column half of Q;
 //   * keys stream through shared memory in tiles of 128 (TMA, 128-byte
-//     swizzle; paged caches use one box per page);
-//   * S = Q K^T goes to TMEM (double buffered, 2 x 128 columns) via
-//     tcgen05.mma issued by one thread; softmax warps read S with
-//     tcgen05.ld, apply the mask from indices, run the online softmax (exp2
-//     on the MUFU), write P (bf16) to shared memory; O += P V accumulates in
-//     TMEM (128 columns);
+//     swizzle; paged caches use one box per page), K and V on separate rings
+//     with separate producer warps;
+//   * two softmax warpgroups take alternate key tiles. Each owns an S buffer
+//     and an O accumulator in TMEM and a P buffer in shared memory, so the
+//     softmax of tile i+1 runs while tile i's P*V runs and tile i+2's Q*K^T
+//     is already queued. The two partial results (O_b, running max m_b, sum
+//     l_b) are merged per row at the end;
+//   * S = Q K^T and O += P V are tcgen05.mma ops issued by one thread; the
+//     softmax reads S with tcgen05.ld, applies the mask from indices, and runs
+//     the online softmax (exp2 on the MUFU, rescaling O only when the running
+//     maximum grows by more than 2^8);
 //   * when the key range is split across CTAs, each writes a normalised
 //     partial (O_i, log2-sum-exp_i) to the workspace and the last CTA to
 //     arrive merges them: O = sum_i 2^(lse_i - lse_max) O_i / sum_i 2^(...).
 //
-// Warp roles (256 threads): warp 0 TMA producer, warp 1 MMA issuer, warp 2
-// TMEM allocator, warp 3 idle, warps 4-7 softmax + epilogue (warp w reads
-// TMEM lanes 32*(w%4) .. +31, i.e. packed rows of that range).
+// Warp roles (384 threads): warp 0 K producer (and Q), warp 1 MMA issuer,
+// warp 2 V producer, warp 3 TMEM allocator, warps 4-7 softmax group 0 (even
+// tiles), warps 8-11 softmax group 1 (odd tiles). Warp w reads TMEM lanes
+// 32*(w%4) .. +31, i.e. the packed rows of that range.
 //
 // Every mbarrier wait is bounded (about 2 s of global time); a wait that
 // gives up records ZARYA_DEVERR_TIMEOUT, raises a CTA-wide abort flag and the
@@ -36,20 +42,20 @@
 namespace zarya {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kStagesK = 3;
+constexpr int kThreads = 384;
+constexpr int kStagesK = 2;
 constexpr int kStagesV = 2;
 constexpr uint32_t kHalfBytes = kBlockN * 64 * 2;   // 128 rows x 128 B
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;     // 32 KB (128 x 128 bf16)
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + kTileBytes;
+constexpr uint32_t kOffP = kOffQ + kTileBytes;                 // 2 buffers
+constexpr uint32_t kOffK = kOffP + 2 * kTileBytes;
 constexpr uint32_t kOffV = kOffK + kStagesK * kTileBytes;
-constexpr uint32_t kOffP = kOffV + kStagesV * kTileBytes;
-constexpr uint32_t kOffBar = kOffP + kTileBytes;
-constexpr uint32_t kTmemCols = 512;                 // S0 [0,128) S1 [128,256) O [256,384)
+constexpr uint32_t kOffBar = kOffV + kStagesV * kTileBytes;
+constexpr uint32_t kTmemCols = 512;  // S0 [0,128) S1 [128,256) O0 [256,384) O1 [384,512)
 constexpr uint32_t kTmemO = 256;
-constexpr uint64_t kWaitNs = 2000000000ull;         // 2 s
-constexpr uint64_t kDrainNs = 100000000ull;         // 100 ms
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
+constexpr uint64_t kDrainNs = 100000000ull;  // 100 ms
 
 struct Bars {
   uint64_t q_full;
@@ -59,9 +65,11 @@ struct Bars {
   uint64_t v_empty[kStagesV];
   uint64_t s_full[2];
   uint64_t s_free[2];
-  uint64_t p_full;
-  uint64_t o_done;
+  uint64_t p_full[2];
+  uint64_t o_done[2];
   uint64_t drain;
+  uint64_t ready;   // split 0: the other splits' partials are published
+  uint64_t done;    // splits > 0: split 0 has read this CTA's partial
   uint32_t tmem_base;
   int abort;
   int last;
@@ -105,6 +113,65 @@ __device__ __forceinline__ uint32_t kmajor_k_offset(int kk) {
   return (kk >> 2) * kHalfBytes + (kk & 3) * 32;
 }
 
+// One producer warp streams one of K or V through its ring.
+__device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, uint64_t* empty,
+                                        int stages, uint32_t ring, const TcParams& p, Bars* bars,
+                                        int b, int kvh, int t_begin, int nt, int kv_end,
+                                        int lane) {
+  const bool paged = p.page_size > 0;
+  const int ppt = paged ? kBlockN / p.page_size : 0;   // pages per tile
+  const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
+  int issued = 0;
+  bool ok = true;
+  for (int i = 0; i < nt; ++i) {
+    const int t = t_begin + i;
+    int page = -1;
+    uint32_t bytes = kTileBytes;
+    if (paged) {
+      const int lp = t * ppt + lane;
+      const bool want = lane < ppt && lp * p.page_size < kv_end;
+      bool bad = false;
+      if (want) {
+        page = p.page_table[static_cast<long long>(b) * p.max_pages + lp];
+        bad = page < 0 || page >= p.n_pages;
+      }
+      if (__any_sync(0xffffffffu, bad)) {
+        if (lane == 0) set_abort(bars, p.err, ZARYA_DEVERR_PAGE_ID);
+        ok = false;
+        break;
+      }
+      bytes = page_bytes * __popc(__ballot_sync(0xffffffffu, want));
+    }
+    const int s = i % stages;
+    bool w = true;
+    if (lane == 0) {
+      w = wait_bar(&empty[s], ((i / stages) & 1) ^ 1, bars, p.err);
+      if (w) mbar_arrive_expect_tx(&full[s], bytes);
+    }
+    if (!__shfl_sync(0xffffffffu, w, 0)) {
+      ok = false;
+      break;
+    }
+    issued = i + 1;
+    const uint32_t dst = ring + s * kTileBytes;
+    if (!paged) {
+      if (lane == 0) {
+        tma_load_4d(dst, map, &full[s], 0, kvh, t * kBlockN, b);
+        tma_load_4d(dst + kHalfBytes, map, &full[s], 64, kvh, t * kBlockN, b);
+      }
+    } else if (page >= 0) {
+      const uint32_t o = lane * p.page_size * 128;
+      tma_load_4d(dst + o, map, &full[s], 0, kvh, 0, page);
+      tma_load_4d(dst + kHalfBytes + o, map, &full[s], 64, kvh, 0, page);
+    }
+  }
+  if (!ok && lane == 0) {
+    // Let this CTA's own copies land before the CTA (and its smem) goes away.
+    for (int i = max(0, issued - stages); i < issued; ++i)
+      mbar_wait(&full[i % stages], (i / stages) & 1, kDrainNs, nullptr);
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                     const __grid_constant__ CUtensorMap map_k,
@@ -122,6 +189,19 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   const int b = bh / p.Hkv;
   const int kvh = bh - b * p.Hkv;
 
+  // ---- set-up that needs no input (overlaps the previous kernel's tail) ----
+  if (warp == 3) {
+    tmem_alloc(&bars->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&map_q);
+    tma_prefetch_map(&map_k);
+    tma_prefetch_map(&map_v);
+  }
+  // Inputs may be written by the kernel launched before this one.
+  grid_dependency_wait();
+
   // ---- per-sequence geometry (uniform over the CTA) ----
   const int P = p.cache_lens[b];
   const int R = p.n_slots[b] * p.slot_len[b];
@@ -133,24 +213,16 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   else if (R <= 0 || R > p.max_rows || row_end - row0 != R || row0 < 0 || row_end > p.total_rows)
     code = ZARYA_DEVERR_ROWS;
   else if (P < 0 || static_cast<long long>(P) + R > p.capacity) code = ZARYA_DEVERR_CAPACITY;
-  if (code != 0) {
-    if (mt == 0 && split == 0 && threadIdx.x == 0) record_error(p.err, code);
-    return;
-  }
   const int rows_per_tile = kBlockM / p.g;
   const int r0 = mt * rows_per_tile;
-  if (r0 >= R) return;
   const int r_hi = min(r0 + rows_per_tile, R) - 1;
   const int kv_end = (mode == ZARYA_MASK_SLOT_CAUSAL) ? P + r_hi + 1 : P + R;
-  const int n_tiles = (kv_end + kBlockN - 1) / kBlockN;
-  const int per_split = (n_tiles + p.splits - 1) / p.splits;
+  const int n_tiles = (code != 0 || kv_end <= 0) ? 1 : (kv_end + kBlockN - 1) / kBlockN;
+  const int per_split = max(1, (n_tiles + p.splits - 1) / p.splits);
   const int active = (n_tiles + per_split - 1) / per_split;
-  if (split >= active) return;
   const int t_begin = split * per_split;
   const int nt = min(n_tiles, t_begin + per_split) - t_begin;
-  const bool paged = p.page_size > 0;
 
-  // ---- set-up ----
   if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
     for (int s = 0; s < kStagesK; ++s) {
@@ -164,115 +236,53 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bars->s_full[s], 1);
       mbar_init(&bars->s_free[s], 4);
+      mbar_init(&bars->p_full[s], 4);
+      mbar_init(&bars->o_done[s], 1);
     }
-    mbar_init(&bars->p_full, 4);
-    mbar_init(&bars->o_done, 1);
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->ready, active > 1 ? active - 1 : 1);
+    mbar_init(&bars->done, 1);
     bars->abort = 0;
     bars->last = 0;
     fence_mbar_init();
-  }
-  if (warp == 2) {
-    tmem_alloc(&bars->tmem_base, kTmemCols);
-    tmem_relinquish();
-  }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_map(&map_q);
-    tma_prefetch_map(&map_k);
-    tma_prefetch_map(&map_v);
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
+  // Exits before the cluster barrier are uniform over a cluster (its CTAs
+  // share the sequence and M-tile and differ only in the split).
+  if (code != 0 || r0 >= R) {
+    if (code != 0 && mt == 0 && split == 0 && threadIdx.x == 0) record_error(p.err, code);
+    grid_launch_dependents();
+    if (warp == 3) tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
+  // Every CTA of the cluster has initialised its barriers before any remote
+  // arrive can target them.
+  if (p.cluster) cluster_sync();
+  if (split >= active) {
+    grid_launch_dependents();
+    if (warp == 3) tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
 
   if (warp == 0) {
-    // ======================= TMA producer =======================
-    int issued_k = 0, issued_v = 0;
-    bool ok = true;
+    // ======================= Q + K producer =======================
     if (lane == 0) {
       mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
       const uint32_t dq = smem_u32(smem + kOffQ);
       tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
       tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
     }
-    const int ppt = paged ? kBlockN / p.page_size : 0;   // pages per tile
-    const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
-    for (int i = 0; i < nt && ok; ++i) {
-      const int t = t_begin + i;
-      // page ids of this tile: lane l < ppt owns page l
-      int page = -1;
-      uint32_t bytes = kTileBytes;
-      if (paged) {
-        const int lp = t * ppt + lane;
-        const bool want = lane < ppt && lp * p.page_size < kv_end;
-        bool bad = false;
-        if (want) {
-          page = p.page_table[static_cast<long long>(b) * p.max_pages + lp];
-          bad = page < 0 || page >= p.n_pages;
-        }
-        if (__any_sync(0xffffffffu, bad)) {
-          if (lane == 0) set_abort(bars, p.err, ZARYA_DEVERR_PAGE_ID);
-          ok = false;
-          break;
-        }
-        bytes = page_bytes * __popc(__ballot_sync(0xffffffffu, want));
-      }
-      // K tile
-      {
-        const int s = i % kStagesK;
-        const uint32_t ph = (i / kStagesK) & 1;
-        bool w = true;
-        if (lane == 0) {
-          w = wait_bar(&bars->k_empty[s], ph ^ 1, bars, p.err);
-          if (w) mbar_arrive_expect_tx(&bars->k_full[s], bytes);
-        }
-        if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
-        issued_k = i + 1;
-        const uint32_t dst = smem_u32(smem + kOffK + s * kTileBytes);
-        if (!paged) {
-          if (lane == 0) {
-            tma_load_4d(dst, &map_k, &bars->k_full[s], 0, kvh, t * kBlockN, b);
-            tma_load_4d(dst + kHalfBytes, &map_k, &bars->k_full[s], 64, kvh, t * kBlockN, b);
-          }
-        } else if (page >= 0) {
-          const uint32_t o = lane * p.page_size * 128;
-          tma_load_4d(dst + o, &map_k, &bars->k_full[s], 0, kvh, 0, page);
-          tma_load_4d(dst + kHalfBytes + o, &map_k, &bars->k_full[s], 64, kvh, 0, page);
-        }
-      }
-      // V tile
-      {
-        const int s = i % kStagesV;
-        const uint32_t ph = (i / kStagesV) & 1;
-        bool w = true;
-        if (lane == 0) {
-          w = wait_bar(&bars->v_empty[s], ph ^ 1, bars, p.err);
-          if (w) mbar_arrive_expect_tx(&bars->v_full[s], bytes);
-        }
-        if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
-        issued_v = i + 1;
-        const uint32_t dst = smem_u32(smem + kOffV + s * kTileBytes);
-        if (!paged) {
-          if (lane == 0) {
-            tma_load_4d(dst, &map_v, &bars->v_full[s], 0, kvh, t * kBlockN, b);
-            tma_load_4d(dst + kHalfBytes, &map_v, &bars->v_full[s], 64, kvh, t * kBlockN, b);
-          }
-        } else if (page >= 0) {
-          const uint32_t o = lane * p.page_size * 128;
-          tma_load_4d(dst + o, &map_v, &bars->v_full[s], 0, kvh, 0, page);
-          tma_load_4d(dst + kHalfBytes + o, &map_v, &bars->v_full[s], 64, kvh, 0, page);
-        }
-      }
-    }
-    if (!ok && lane == 0) {
-      // Let this CTA's own copies land before the CTA (and its smem) goes away.
-      for (int i = max(0, issued_k - kStagesK); i < issued_k; ++i)
-        mbar_wait(&bars->k_full[i % kStagesK], (i / kStagesK) & 1, kDrainNs, nullptr);
-      for (int i = max(0, issued_v - kStagesV); i < issued_v; ++i)
-        mbar_wait(&bars->v_full[i % kStagesV], (i / kStagesV) & 1, kDrainNs, nullptr);
+    produce(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars, b,
+            kvh, t_begin, nt, kv_end, lane);
+    if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
       mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
-    }
+  } else if (warp == 2) {
+    // ======================= V producer =======================
+    produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
+            kvh, t_begin, nt, kv_end, lane);
   } else if (warp == 1) {
     // ======================= MMA issuer (one thread) =======================
     if (lane == 0) {
@@ -280,28 +290,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       bool any_mma = false;
       tc_fence_after();
       const uint32_t q_addr = smem_u32(smem + kOffQ);
-      const uint32_t p_addr = smem_u32(smem + kOffP);
-      auto issue_pv = [&](int j) -> bool {
-        const int sv = j % kStagesV;
-        if (!wait_bar(&bars->p_full, j & 1, bars, p.err)) return false;
-        if (!wait_bar(&bars->v_full[sv], (j / kStagesV) & 1, bars, p.err)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(smem + kOffV + sv * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = sdesc_sw128(p_addr + kmajor_k_offset(kk), 16, 1024);
-          const uint64_t bd = sdesc_sw128(v_addr + kk * 2048, kHalfBytes, 1024);
-          tc_mma_ss(tmem + kTmemO, ad, bd, kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
-        }
-        tc_commit(&bars->o_done);
-        tc_commit(&bars->v_empty[sv]);
-        return true;
-      };
-      for (int i = 0; i < nt && ok; ++i) {
+      auto issue_qk = [&](int i) -> bool {
         const int s = i % kStagesK;
         const int sb = i & 1;
-        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) { ok = false; break; }
-        if (!wait_bar(&bars->s_free[sb], ((i >> 1) & 1) ^ 1, bars, p.err)) { ok = false; break; }
+        const int j = i >> 1;
+        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
+        if (j > 0 && !wait_bar(&bars->s_free[sb], (j - 1) & 1, bars, p.err)) return false;
         tc_fence_after();
         const uint32_t k_addr = smem_u32(smem + kOffK + s * kTileBytes);
 #pragma unroll
@@ -313,9 +307,34 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         any_mma = true;
         tc_commit(&bars->s_full[sb]);
         tc_commit(&bars->k_empty[s]);
-        if (i > 0 && !issue_pv(i - 1)) { ok = false; break; }
+        return true;
+      };
+      auto issue_pv = [&](int i) -> bool {
+        const int sv = i % kStagesV;
+        const int sb = i & 1;
+        const int j = i >> 1;
+        if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
+        if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
+        tc_fence_after();
+        const uint32_t p_addr = smem_u32(smem + kOffP + sb * kTileBytes);
+        const uint32_t v_addr = smem_u32(smem + kOffV + sv * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t ad = sdesc_sw128(p_addr + kmajor_k_offset(kk), 16, 1024);
+          const uint64_t bd = sdesc_sw128(v_addr + kk * 2048, kHalfBytes, 1024);
+          tc_mma_ss(tmem + kTmemO + sb * 128, ad, bd, kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+        }
+        any_mma = true;
+        tc_commit(&bars->o_done[sb]);
+        tc_commit(&bars->v_empty[sv]);
+        return true;
+      };
+      if (ok) ok = issue_qk(0);
+      if (ok && nt > 1) ok = issue_qk(1);
+      for (int i = 0; i < nt && ok; ++i) {
+        if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
+        if (!issue_pv(i)) { ok = false; break; }
       }
-      if (ok && nt > 0) ok = issue_pv(nt - 1);
       if (!ok && any_mma) {
         tc_commit(&bars->drain);
         mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
@@ -323,46 +342,49 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     }
   } else if (warp >= 4) {
     // ======================= softmax + epilogue =======================
+    const int grp = (warp - 4) >> 2;                // 0: even tiles, 1: odd tiles
     const int wq = warp & 3;
     const int m = wq * 32 + lane;                   // packed row = TMEM lane
     const int r = r0 + m / p.g;
     const int h = kvh * p.g + (m - (m / p.g) * p.g);
     const bool row_ok = r <= r_hi;
     const int limit = !row_ok ? kv_end : (mode == ZARYA_MASK_SLOT_CAUSAL ? P + r + 1 : P + R);
-    const uint32_t t_lane = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    const uint32_t t_row = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    const uint32_t t_s = t_row + grp * 128;
+    const uint32_t t_o = t_row + kTmemO + grp * 128;
     const float sl2 = p.scale_log2;
     float m_run = -INFINITY;  // running max, in scaled log2 units
     float l_run = 0.f;
     bool ok = true;
-    uint8_t* sp = smem + kOffP;
+    uint8_t* prow = smem + kOffP + grp * kTileBytes + (m >> 3) * 1024 + (m & 7) * 128;
 
-    for (int i = 0; i < nt; ++i) {
+    for (int i = grp; i < nt; i += 2) {
+      const int j = i >> 1;
       const int c0 = (t_begin + i) * kBlockN;
-      const int sb = i & 1;
-      if (ok) ok = wait_bar(&bars->s_full[sb], (i >> 1) & 1, bars, p.err);
+      if (ok) ok = wait_bar(&bars->s_full[grp], j & 1, bars, p.err);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       float s[128];
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        float v[32];
-        tmem_ld_32x32b_x32(t_lane + sb * 128 + ch * 32, v);
-#pragma unroll
-        for (int x = 0; x < 32; ++x) s[ch * 32 + x] = v[x];
-      }
+      tmem_ld_32x32b_x128(t_s, s);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->s_free[sb]);
+      if (lane == 0) mbar_arrive(&bars->s_free[grp]);
 
       if (c0 + kBlockN > limit) {
 #pragma unroll
         for (int x = 0; x < 128; ++x)
           if (c0 + x >= limit) s[x] = -INFINITY;
       }
-      float mx = -INFINITY;
+      float mx[8];
 #pragma unroll
-      for (int x = 0; x < 128; ++x) mx = fmaxf(mx, s[x]);
-      const float m_new = fmaxf(m_run, mx * sl2);
+      for (int k = 0; k < 8; ++k) mx[k] = s[k];
+#pragma unroll
+      for (int x = 8; x < 128; x += 8)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], s[x + k]);
+      const float mt4 = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+      const float mt8 = fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]));
+      const float m_new = fmaxf(m_run, fmaxf(mt4, mt8) * sl2);
       const bool need = m_new > m_run + 8.0f;
       const bool warp_need = __any_sync(0xffffffffu, need);
       float alpha = 1.f;
@@ -372,17 +394,25 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         l_run *= alpha;
       }
       const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-      uint32_t pk[64];
-      float rs = 0.f;
-#pragma unroll
-      for (int x = 0; x < 128; x += 2) {
-        const float p0 = fast_exp2(fmaf(s[x], sl2, -m_use));
-        const float p1 = fast_exp2(fmaf(s[x + 1], sl2, -m_use));
-        rs += p0 + p1;
-        pk[x >> 1] = pack_bf16(p0, p1);
-      }
-      l_run += rs;
 
+      // This group's previous P*V must be done before its P buffer and O
+      // accumulator are touched again.
+      if (j > 0) {
+        if (ok) ok = wait_bar(&bars->o_done[grp], (j - 1) & 1, bars, p.err);
+        tc_fence_after();
+      }
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      if (warp_need && j > 0) {
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          float v[32];
+          const uint32_t a = t_o + ch * 32;
+          tmem_ld_32x32b_x32(a, v);
+#pragma unroll
+          for (int x = 0; x < 32; ++x) v[x] *= alpha;
+          tmem_st_32x32b_x32(a, v);
+        }
+      }
       // Keys at or past kv_end in the last tile: their V rows (stale smem,
       // unloaded pages or another sequence's cache) must be exact zeros, or a
       // NaN there would poison P*V even with P = 0.
@@ -399,126 +429,212 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           }
         }
       }
-      // P of the previous tile must have been consumed (and O be final for
-      // the rescale) before P is overwritten.
-      if (i > 0) {
-        if (ok) ok = wait_bar(&bars->o_done, (i - 1) & 1, bars, p.err);
-        tc_fence_after();
-      }
-      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-      if (warp_need && i > 0) {
-#pragma unroll
-        for (int ch = 0; ch < 4; ++ch) {
-          float v[32];
-          const uint32_t a = t_lane + kTmemO + ch * 32;
-          tmem_ld_32x32b_x32(a, v);
-#pragma unroll
-          for (int x = 0; x < 32; ++x) v[x] *= alpha;
-          tmem_st_32x32b_x32(a, v);
-        }
-      }
-      uint8_t* prow = sp + (m >> 3) * 1024 + (m & 7) * 128;
+      float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
 #pragma unroll
       for (int c16 = 0; c16 < 16; ++c16) {
+        float e[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) e[k] = fast_exp2(fmaf(s[c16 * 8 + k], sl2, -m_use));
+        rs0 += e[0] + e[4];
+        rs1 += e[1] + e[5];
+        rs2 += e[2] + e[6];
+        rs3 += e[3] + e[7];
         const uint32_t off = (c16 >> 3) * kHalfBytes + ((((c16 & 7) ^ (m & 7))) << 4);
         *reinterpret_cast<uint4*>(prow + off) =
-            make_uint4(pk[c16 * 4 + 0], pk[c16 * 4 + 1], pk[c16 * 4 + 2], pk[c16 * 4 + 3]);
+            make_uint4(pack_bf16(e[0], e[1]), pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]),
+                       pack_bf16(e[6], e[7]));
       }
+      l_run += (rs0 + rs1) + (rs2 + rs3);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->p_full);
+      if (lane == 0) mbar_arrive(&bars->p_full[grp]);
     }
 
-    // ---- epilogue ----
-    if (ok) ok = wait_bar(&bars->o_done, (nt - 1) & 1, bars, p.err);
+    // ---- epilogue: merge the two groups' partial results per row ----
+    const int n0 = (nt + 1) >> 1;   // tiles of group 0
+    const int n1 = nt >> 1;         // tiles of group 1
+    const int n_mine = grp == 0 ? n0 : n1;
+    if (n_mine > 0) {
+      if (ok) ok = wait_bar(&bars->o_done[grp], (n_mine - 1) & 1, bars, p.err);
+    }
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_after();
+    // Both P buffers are idle now (each group waited for its last P*V): they
+    // carry the (max, sum) exchange between the groups.
+    float* xch = reinterpret_cast<float*>(smem + kOffP + grp * kTileBytes);
+    xch[m] = m_run;
+    xch[128 + m] = l_run;
+    tc_fence_before();
+    named_bar_sync(1, 256);
+    tc_fence_after();
+    const float* x0 = reinterpret_cast<const float*>(smem + kOffP);
+    const float* x1 = reinterpret_cast<const float*>(smem + kOffP + kTileBytes);
+    const float mA = x0[m], lA = x0[128 + m];
+    const float mB = x1[m], lB = x1[128 + m];
+    const float mT = fmaxf(mA, mB);
+    const float aA = (mA == -INFINITY) ? 0.f : fast_exp2(mA - mT);
+    const float aB = (mB == -INFINITY) ? 0.f : fast_exp2(mB - mT);
+    const float lT = aA * lA + aB * lB;
+    const float inv = (lT > 0.f) ? 1.f / lT : 0.f;
+    const float wA = aA * inv, wB = aB * inv;
     const long long unit = static_cast<long long>(bh) * p.m_tiles + mt;
+    const int col0 = grp * 64;   // group g finishes columns [64g, 64g + 64)
+    grid_launch_dependents();
+
+    // This CTA's result for its 64 columns of row m, normalised.
+    float o[64];
+#pragma unroll
+    for (int ch = 0; ch < 2; ++ch) {
+      float va[32], vb[32];
+      if (ok && n0 > 0) tmem_ld_32x32b_x32(t_row + kTmemO + col0 + ch * 32, va);
+      else {
+#pragma unroll
+        for (int x = 0; x < 32; ++x) va[x] = 0.f;
+      }
+      if (ok && n1 > 0) tmem_ld_32x32b_x32(t_row + kTmemO + 128 + col0 + ch * 32, vb);
+      else {
+#pragma unroll
+        for (int x = 0; x < 32; ++x) vb[x] = 0.f;
+      }
+#pragma unroll
+      for (int x = 0; x < 32; ++x) o[ch * 32 + x] = wA * va[x] + wB * vb[x];
+    }
+    __nv_bfloat16* out_row = reinterpret_cast<__nv_bfloat16*>(p.out) +
+                             (static_cast<long long>(row0 + r) * p.Hq + h) * kHeadDim + col0;
+    auto store_out = [&](const float (&v)[64], float scale) {
+      uint4* d4 = reinterpret_cast<uint4*>(out_row);
+#pragma unroll
+      for (int x = 0; x < 8; ++x)
+        d4[x] = make_uint4(pack_bf16(v[8 * x + 0] * scale, v[8 * x + 1] * scale),
+                           pack_bf16(v[8 * x + 2] * scale, v[8 * x + 3] * scale),
+                           pack_bf16(v[8 * x + 4] * scale, v[8 * x + 5] * scale),
+                           pack_bf16(v[8 * x + 6] * scale, v[8 * x + 7] * scale));
+    };
     if (active == 1) {
-      const float inv = (l_run > 0.f) ? 1.f / l_run : 0.f;
-      __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.out) +
-                           (static_cast<long long>(row0 + r) * p.Hq + h) * kHeadDim;
-#pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        float v[32];
-        if (ok) tmem_ld_32x32b_x32(t_lane + kTmemO + ch * 32, v);
+      if (ok && row_ok) store_out(o, 1.f);
+    } else if (p.cluster) {
+      // Split key range, splits of this tile in one cluster: splits > 0
+      // publish their normalised partial (O_s, lse_s) in their own shared
+      // memory (the K ring, idle now) and signal split 0, which reads them
+      // through distributed shared memory and merges in split order:
+      //   O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M),  M = max_s lse_s.
+      const float lse_own = (lT > 0.f) ? mT + __log2f(lT) : -INFINITY;
+      const uint32_t xbuf = smem_u32(smem + kOffK);   // [128 rows][512 B], 16-B chunks swizzled
+      const uint32_t lbuf = smem_u32(smem + kOffV);   // [128] fp32
+      const uint32_t xrow = xbuf + m * 512;
+      const int c_base = col0 >> 2;                  // first 16-byte chunk of my columns
+      if (split > 0) {
         if (ok && row_ok) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + ch * 32);
 #pragma unroll
-          for (int x = 0; x < 4; ++x)
-            d4[x] = make_uint4(pack_bf16(v[8 * x + 0] * inv, v[8 * x + 1] * inv),
-                               pack_bf16(v[8 * x + 2] * inv, v[8 * x + 3] * inv),
-                               pack_bf16(v[8 * x + 4] * inv, v[8 * x + 5] * inv),
-                               pack_bf16(v[8 * x + 6] * inv, v[8 * x + 7] * inv));
+          for (int c = 0; c < 16; ++c) {
+            const uint32_t a = xrow + ((((c_base + c) ^ (m & 31))) << 4);
+            asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(o[4 * c]),
+                         "f"(o[4 * c + 1]), "f"(o[4 * c + 2]), "f"(o[4 * c + 3])
+                         : "memory");
+          }
+          if (grp == 0)
+            asm volatile("st.shared.f32 [%0], %1;" ::"r"(lbuf + m * 4), "f"(lse_own) : "memory");
         }
+        named_bar_sync(1, 256);
+        if (grp == 0 && m == 0) {
+          if (*reinterpret_cast<volatile int*>(&bars->abort) == 0) {
+            mbar_arrive_remote(mapa_shared(smem_u32(&bars->ready), 0));
+            // split 0 reads this CTA's shared memory: stay until it is done
+            if (!mbar_wait_cluster(&bars->done, 0, kWaitNs, nullptr))
+              set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
+          }
+        }
+        named_bar_sync(1, 256);
+      } else {
+        if (grp == 0 && m == 0) {
+          const bool got = mbar_wait_cluster(&bars->ready, 0, kWaitNs, &bars->abort);
+          if (!got) set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
+          bars->last = got ? 1 : 0;
+        }
+        named_bar_sync(1, 256);
+        if (*reinterpret_cast<volatile int*>(&bars->last) && ok && row_ok) {
+          float M = lse_own;
+          float S = (lse_own == -INFINITY) ? 0.f : 1.f;
+          for (int sp = 1; sp < active; ++sp) {
+            const float ls = ld_shared_cluster_f32(mapa_shared(lbuf + m * 4, sp));
+            const uint32_t rx = mapa_shared(xrow, sp);
+            float4 v[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c)
+              v[c] = ld_shared_cluster_f4(rx + ((((c_base + c) ^ (m & 31))) << 4));
+            const float Mn = fmaxf(M, ls);
+            const float a = (M == -INFINITY) ? 0.f : fast_exp2(M - Mn);
+            const float c2 = (ls == -INFINITY) ? 0.f : fast_exp2(ls - Mn);
+            S = S * a + c2;
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              o[4 * c + 0] = o[4 * c + 0] * a + c2 * v[c].x;
+              o[4 * c + 1] = o[4 * c + 1] * a + c2 * v[c].y;
+              o[4 * c + 2] = o[4 * c + 2] * a + c2 * v[c].z;
+              o[4 * c + 3] = o[4 * c + 3] * a + c2 * v[c].w;
+            }
+            M = Mn;
+          }
+          store_out(o, S > 0.f ? 1.f / S : 0.f);
+        }
+        named_bar_sync(1, 256);
+        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->last))
+          for (int sp = 1; sp < active; ++sp)
+            mbar_arrive_remote(mapa_shared(smem_u32(&bars->done), sp));
       }
     } else {
-      const float inv = (l_run > 0.f) ? 1.f / l_run : 0.f;
-      const long long slot = (unit * p.splits + split) * kBlockM + m;
-      float* po = p.ws_o + slot * kHeadDim;
+      // Split key range beyond a cluster: every split writes its partial to
+      // the workspace, takes a ticket, and the last one merges all of them in
+      // split order (so the result does not depend on the arrival order).
+      const float lse_own = (lT > 0.f) ? mT + __log2f(lT) : -INFINITY;
+      const long long own = (unit * p.splits + split) * kBlockM + m;
+      if (ok && row_ok) {
+        float4* d4 = reinterpret_cast<float4*>(p.ws_o + own * kHeadDim + col0);
 #pragma unroll
-      for (int ch = 0; ch < 4; ++ch) {
-        float v[32];
-        if (ok) tmem_ld_32x32b_x32(t_lane + kTmemO + ch * 32, v);
-        if (ok && row_ok) {
-          float4* d4 = reinterpret_cast<float4*>(po + ch * 32);
-#pragma unroll
-          for (int x = 0; x < 8; ++x)
-            d4[x] = make_float4(v[4 * x] * inv, v[4 * x + 1] * inv, v[4 * x + 2] * inv,
-                                v[4 * x + 3] * inv);
-        }
+        for (int x = 0; x < 16; ++x)
+          d4[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+        if (grp == 0) p.ws_lse[own] = lse_own;
       }
-      if (row_ok) p.ws_lse[slot] = (l_run > 0.f) ? m_run + __log2f(l_run) : -INFINITY;
       __threadfence();
-      named_bar_sync(1, 128);
-      if (m == 0) {
+      named_bar_sync(1, 256);
+      if (grp == 0 && m == 0) {
         int last = 0;
-        if (*reinterpret_cast<volatile int*>(&bars->abort) == 0) {
-          const int prev = atomicAdd(&p.ws_count[unit], 1);
-          last = (prev == active - 1);
-        }
+        if (*reinterpret_cast<volatile int*>(&bars->abort) == 0)
+          last = (atomicAdd(&p.ws_count[unit], 1) == active - 1) ? 1 : 0;
         bars->last = last;
       }
-      named_bar_sync(1, 128);
+      named_bar_sync(1, 256);
       if (*reinterpret_cast<volatile int*>(&bars->last)) {
         __threadfence();
-        if (row_ok) {
-          const long long base = unit * p.splits * kBlockM + m;
-          float lmax = -INFINITY;
-          for (int sp2 = 0; sp2 < active; ++sp2)
-            lmax = fmaxf(lmax, __ldcg(p.ws_lse + base + sp2 * kBlockM));
-          float acc[kHeadDim];
+        if (ok && row_ok) {
+          float M = -INFINITY, S = 0.f;
 #pragma unroll
-          for (int d = 0; d < kHeadDim; ++d) acc[d] = 0.f;
-          float wsum = 0.f;
-          for (int sp2 = 0; sp2 < active; ++sp2) {
-            const float lse = __ldcg(p.ws_lse + base + sp2 * kBlockM);
-            const float w = (lse == -INFINITY) ? 0.f : fast_exp2(lse - lmax);
-            wsum += w;
-            const float4* src =
-                reinterpret_cast<const float4*>(p.ws_o + (base + sp2 * kBlockM) * kHeadDim);
+          for (int x = 0; x < 64; ++x) o[x] = 0.f;
+          for (int sp = 0; sp < active; ++sp) {
+            const long long slot = (unit * p.splits + sp) * kBlockM + m;
+            const float ls = __ldcg(p.ws_lse + slot);
+            const float4* src = reinterpret_cast<const float4*>(p.ws_o + slot * kHeadDim + col0);
+            float4 v[16];
 #pragma unroll
-            for (int d4 = 0; d4 < kHeadDim / 4; ++d4) {
-              const float4 o = __ldcg(src + d4);
-              acc[4 * d4 + 0] = fmaf(w, o.x, acc[4 * d4 + 0]);
-              acc[4 * d4 + 1] = fmaf(w, o.y, acc[4 * d4 + 1]);
-              acc[4 * d4 + 2] = fmaf(w, o.z, acc[4 * d4 + 2]);
-              acc[4 * d4 + 3] = fmaf(w, o.w, acc[4 * d4 + 3]);
+            for (int x = 0; x < 16; ++x) v[x] = __ldcg(src + x);
+            const float Mn = fmaxf(M, ls);
+            const float a = (M == -INFINITY) ? 0.f : fast_exp2(M - Mn);
+            const float c2 = (ls == -INFINITY) ? 0.f : fast_exp2(ls - Mn);
+            S = S * a + c2;
+#pragma unroll
+            for (int x = 0; x < 16; ++x) {
+              o[4 * x + 0] = o[4 * x + 0] * a + c2 * v[x].x;
+              o[4 * x + 1] = o[4 * x + 1] * a + c2 * v[x].y;
+              o[4 * x + 2] = o[4 * x + 2] * a + c2 * v[x].z;
+              o[4 * x + 3] = o[4 * x + 3] * a + c2 * v[x].w;
             }
+            M = Mn;
           }
-          const float inv2 = 1.f / wsum;
-          uint4* d4 = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) +
-                                               (static_cast<long long>(row0 + r) * p.Hq + h) *
-                                                   kHeadDim);
-#pragma unroll
-          for (int x = 0; x < kHeadDim / 8; ++x)
-            d4[x] = make_uint4(pack_bf16(acc[8 * x + 0] * inv2, acc[8 * x + 1] * inv2),
-                               pack_bf16(acc[8 * x + 2] * inv2, acc[8 * x + 3] * inv2),
-                               pack_bf16(acc[8 * x + 4] * inv2, acc[8 * x + 5] * inv2),
-                               pack_bf16(acc[8 * x + 6] * inv2, acc[8 * x + 7] * inv2));
+          store_out(o, S > 0.f ? 1.f / S : 0.f);
         }
-        if (m == 0) atomicExch(&p.ws_count[unit], 0);
+        named_bar_sync(1, 256);
+        if (grp == 0 && m == 0) atomicExch(&p.ws_count[unit], 0);
       }
     }
   }
@@ -526,7 +642,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   // ---- teardown ----
   tc_fence_before();
   __syncthreads();
-  if (warp == 2) {
+  if (warp == 3) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -549,9 +665,24 @@ cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
-  dim3 grid(p.m_tiles, p.splits, p.B * p.Hkv);
-  slot_attn_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(map_q, map_k, map_v, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[2]{};
+  cfg.gridDim = dim3(p.m_tiles, p.splits, p.B * p.Hkv);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 1;
+  if (p.cluster) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 1;
+    attr[1].val.clusterDim.y = p.splits;
+    attr[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
+  }
+  cfg.attrs = attr;
+  return cudaLaunchKernelEx(&cfg, slot_attn_tc_kernel, map_q, map_k, map_v, p);
 }
 
 }  // namespace zarya

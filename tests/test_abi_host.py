@@ -97,19 +97,23 @@ def test_workspace_size_is_zero_for_invalid_or_fp32(lib):
 
 
 def test_workspace_size_for_forced_splits(lib):
-    # 2 sequences x 8 KV heads x 1 M-tile, 3 splits: partial O + lse + counters
-    d = _desc(kv_splits=3, cache_capacity=512)
-    n = 2 * 8 * 1 * 3 * 128
+    # 2 sequences x 8 KV heads x 1 M-tile, 10 splits (more than a cluster
+    # holds, so they merge through the workspace): partial O + lse + counters
+    d = _desc(kv_splits=10, cache_capacity=2048)
+    n = 2 * 8 * 1 * 10 * 128
     expect = n * 128 * 4
     expect = (expect + 255) // 256 * 256 + n * 4
     expect = (expect + 255) // 256 * 256 + 16 * 4
     expect = (expect + 255) // 256 * 256
     assert lib.zarya_slot_attn_workspace_size(ctypes.byref(d)) == expect
-    assert lib.zarya_slot_attn_workspace_size(ctypes.byref(_desc(kv_splits=1))) == 0
+    # up to 8 splits merge inside a cluster and need no workspace
+    for s in (1, 2, 8):
+        d = _desc(kv_splits=s, cache_capacity=2048)
+        assert lib.zarya_slot_attn_workspace_size(ctypes.byref(d)) == 0
 
 
 def test_attention_requires_large_enough_workspace(lib):
-    d = _desc(kv_splits=2)
+    d = _desc(kv_splits=10, cache_capacity=2048)
     need = lib.zarya_slot_attn_workspace_size(ctypes.byref(d))
     assert need > 0
     # validation of the workspace happens after device selection, which needs

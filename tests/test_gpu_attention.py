@@ -67,8 +67,9 @@ def test_reduced_workload_matches_oracle_everywhere(zs, oracle_mod, name, mode):
                                        ("ragged_mid", None)])
 @pytest.mark.parametrize("splits", [1, 2, 3, 7])
 def test_split_kv_merge_matches_oracle(zs, oracle_mod, name, mode, splits):
-    """Forcing the key range to be split n ways (partials merged in-kernel by
-    the last CTA to arrive) still matches the oracle."""
+    """Forcing the key range to be split n ways (up to 8 splits form a
+    thread-block cluster and merge through distributed shared memory) still
+    matches the oracle."""
     w = wl.make(name, small=True)
     db = _run(zs, w, mode, kv_splits=splits)
     kc, vc = oracle_staged(oracle_mod, w)
@@ -77,12 +78,50 @@ def test_split_kv_merge_matches_oracle(zs, oracle_mod, name, mode, splits):
     assert ok, f"{name} splits={splits}: max|err|={err:.3e}"
 
 
-def test_workspace_counters_return_to_zero(zs):
-    """The split merge leaves its arrival counters at zero, so a workspace
-    can be reused: two calls in a row give identical results."""
-    w = wl.make("decode_small", small=True)
+@pytest.mark.parametrize("name,small,override,splits", [("long_ctx", True, {}, 9),
+                                                        ("long_ctx", True, {}, 13),
+                                                        ("decode_small", False, {"B": 2}, 17)])
+def test_workspace_merge_beyond_a_cluster_matches_oracle(zs, oracle_mod, name, small, override,
+                                                         splits):
+    """More than 8 key splits merge through the workspace (last CTA to arrive,
+    in split order) instead of a cluster; still matches the oracle."""
     session, zb = zs
-    db = session.upload(w, "cuda", kv_splits=3)
+    w = wl.make(name, small=small, **override)
+    for mode in (0, 1):
+        db = session.upload(w, "cuda", kv_splits=splits, mask_mode=mode)
+        assert zb.workspace_size(db.desc) > 0
+        db.stage()
+        db.attend()
+        torch.cuda.synchronize()
+        assert zb.check_device_error() == 0
+        kc, vc = oracle_staged(oracle_mod, w)
+        sel = sample_rows(w, 96, seed=3)
+        ref = oracle_rows(oracle_mod, w, kc, vc, sel, mode)
+        ok, err, _ = tolerance_ok(gather_rows(db.out, w, sel), ref, w.dtype)
+        assert ok, f"{name} splits={splits} mode={mode}: max|err|={err:.3e}"
+
+
+@pytest.mark.parametrize("splits", [2, 3, 17])
+def test_split_merge_is_bitwise_deterministic(zs, splits):
+    """The merged result does not depend on which split finishes first."""
+    session, zb = zs
+    w = wl.make("decode_small", B=2)
+    outs = []
+    for _ in range(3):
+        db = session.upload(w, "cuda", kv_splits=splits)
+        db.stage()
+        db.attend()
+        torch.cuda.synchronize()
+        outs.append(db.out.clone())
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+def test_workspace_counters_return_to_zero(zs):
+    """The workspace merge leaves its arrival counters at zero, so a workspace
+    can be reused: two calls in a row give identical results."""
+    w = wl.make("decode_small", B=2)
+    session, zb = zs
+    db = session.upload(w, "cuda", kv_splits=12)
     db.stage()
     db.attend()
     first = db.out.clone()
@@ -150,3 +189,33 @@ def test_full_size_sampled_rows_match_oracle(zs, oracle_mod, name, mode):
     got = gather_rows(out, w, sel)
     ok, err, scale = tolerance_ok(got, ref, w.dtype)
     assert ok, f"{name} mode={mode}: max|err|={err:.3e} max|ref|={scale:.3f}"
+
+
+def test_cuda_graph_capture_of_a_step_matches_eager(zs):
+    """A whole step (stage, attention, commit) captured into a CUDA graph and
+    replayed gives the same output bits and lengths as eager calls."""
+    session, zb = zs
+    w = wl.make("decode_small", small=True)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        eager = session.upload(w, "cuda", kv_splits=2)
+        eager.stage(s)
+        eager.attend(s)
+        eager.commit(s)
+        db = session.upload(w, "cuda", kv_splits=2)
+        db.stage(s)      # warm-up outside the capture
+        db.attend(s)
+    torch.cuda.synchronize()
+    db.cache_lens.copy_(torch.as_tensor(w.cache_lens))
+    db.out.zero_()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        db.stage(s)
+        db.attend(s)
+        db.commit(s)
+    g.replay()
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    assert torch.equal(db.out, eager.out)
+    assert torch.equal(db.cache_lens, eager.cache_lens)
