@@ -13,14 +13,19 @@
 //     swizzle; paged caches use one box per page), K and V on separate rings
 //     with separate producer warps;
 //   * two softmax warpgroups take alternate key tiles. Each owns an S buffer
-//     and an O accumulator in TMEM and a P buffer in shared memory, so the
-//     softmax of tile i+1 runs while tile i's P*V runs and tile i+2's Q*K^T
-//     is already queued. The two partial results (O_b, running max m_b, sum
-//     l_b) are merged per row at the end;
-//   * S = Q K^T and O += P V are tcgen05.mma ops issued by one thread; the
-//     softmax reads S with tcgen05.ld, applies the mask from indices, and runs
-//     the online softmax (exp2 on the MUFU, rescaling O only when the running
-//     maximum grows by more than 2^8);
+//     and an O accumulator in TMEM; P (bf16) is written back over the first
+//     half of its S buffer and P*V takes it straight from TMEM, so shared
+//     memory holds only Q and the K/V rings (3 stages each). The softmax of
+//     tile i+1 runs while tile i's P*V and tile i+2's Q*K^T run. The two
+//     partial results (O_b, running max m_b, sum l_b) are merged per row at
+//     the end;
+//   * S = Q K^T and O += P V are tcgen05.mma ops issued by one thread, in the
+//     order Q*K^T(0), Q*K^T(1), then P*V(i), Q*K^T(i+2) for each i: the
+//     tensor pipe runs one thread's MMAs in issue order, so P*V(i) has read
+//     P(i) before Q*K^T(i+2) overwrites that buffer, and a completed Q*K^T(i)
+//     implies P*V(i-2) is complete too. The softmax reads S with tcgen05.ld,
+//     applies the mask from indices, and runs the online softmax (exp2 on the
+//     MUFU, rescaling O only when the running maximum grows by more than 2^8);
 //   * when the key range is split across CTAs, each writes a normalised
 //     partial (O_i, log2-sum-exp_i) to the workspace and the last CTA to
 //     arrive merges them: O = sum_i 2^(lse_i - lse_max) O_i / sum_i 2^(...).
@@ -43,16 +48,15 @@ namespace zarya {
 namespace {
 
 constexpr int kThreads = 384;
-constexpr int kStagesK = 2;
-constexpr int kStagesV = 2;
+constexpr int kStagesK = 3;
+constexpr int kStagesV = 3;
 constexpr uint32_t kHalfBytes = kBlockN * 64 * 2;   // 128 rows x 128 B
 constexpr uint32_t kTileBytes = 2 * kHalfBytes;     // 32 KB (128 x 128 bf16)
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffP = kOffQ + kTileBytes;                 // 2 buffers
-constexpr uint32_t kOffK = kOffP + 2 * kTileBytes;
+constexpr uint32_t kOffK = kOffQ + kTileBytes;
 constexpr uint32_t kOffV = kOffK + kStagesK * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStagesV * kTileBytes;
-constexpr uint32_t kTmemCols = 512;  // S0 [0,128) S1 [128,256) O0 [256,384) O1 [384,512)
+constexpr uint32_t kTmemCols = 512;  // S0/P0 [0,128) S1/P1 [128,256) O0 [256,384) O1 [384,512)
 constexpr uint32_t kTmemO = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
 constexpr uint64_t kDrainNs = 100000000ull;  // 100 ms
@@ -64,7 +68,6 @@ struct Bars {
   uint64_t v_full[kStagesV];
   uint64_t v_empty[kStagesV];
   uint64_t s_full[2];
-  uint64_t s_free[2];
   uint64_t p_full[2];
   uint64_t o_done[2];
   uint64_t drain;
@@ -235,7 +238,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bars->s_full[s], 1);
-      mbar_init(&bars->s_free[s], 4);
       mbar_init(&bars->p_full[s], 4);
       mbar_init(&bars->o_done[s], 1);
     }
@@ -293,9 +295,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       auto issue_qk = [&](int i) -> bool {
         const int s = i % kStagesK;
         const int sb = i & 1;
-        const int j = i >> 1;
         if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
-        if (j > 0 && !wait_bar(&bars->s_free[sb], (j - 1) & 1, bars, p.err)) return false;
         tc_fence_after();
         const uint32_t k_addr = smem_u32(smem + kOffK + s * kTileBytes);
 #pragma unroll
@@ -316,13 +316,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
         if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
         tc_fence_after();
-        const uint32_t p_addr = smem_u32(smem + kOffP + sb * kTileBytes);
         const uint32_t v_addr = smem_u32(smem + kOffV + sv * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = sdesc_sw128(p_addr + kmajor_k_offset(kk), 16, 1024);
           const uint64_t bd = sdesc_sw128(v_addr + kk * 2048, kHalfBytes, 1024);
-          tc_mma_ss(tmem + kTmemO + sb * 128, ad, bd, kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_ts(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, bd, kIdescPV,
+                    (j > 0 || kk > 0) ? 1u : 0u);
         }
         any_mma = true;
         tc_commit(&bars->o_done[sb]);
@@ -332,8 +331,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       if (ok) ok = issue_qk(0);
       if (ok && nt > 1) ok = issue_qk(1);
       for (int i = 0; i < nt && ok; ++i) {
-        if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
         if (!issue_pv(i)) { ok = false; break; }
+        if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
       }
       if (!ok && any_mma) {
         tc_commit(&bars->drain);
@@ -356,7 +355,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     float m_run = -INFINITY;  // running max, in scaled log2 units
     float l_run = 0.f;
     bool ok = true;
-    uint8_t* prow = smem + kOffP + grp * kTileBytes + (m >> 3) * 1024 + (m & 7) * 128;
 
     for (int i = grp; i < nt; i += 2) {
       const int j = i >> 1;
@@ -366,9 +364,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       tc_fence_after();
       float s[128];
       tmem_ld_32x32b_x128(t_s, s);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->s_free[grp]);
 
       if (c0 + kBlockN > limit) {
 #pragma unroll
@@ -395,13 +390,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       }
       const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
 
-      // This group's previous P*V must be done before its P buffer and O
-      // accumulator are touched again.
-      if (j > 0) {
-        if (ok) ok = wait_bar(&bars->o_done[grp], (j - 1) & 1, bars, p.err);
-        tc_fence_after();
-      }
-      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      // O may be rescaled here: S(i) being complete means this group's
+      // previous P*V (issued before Q*K^T(i)) is complete as well.
       if (warp_need && j > 0) {
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
@@ -429,23 +419,29 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           }
         }
       }
+      // P = 2^(s * scale * log2 e - m) as packed bf16 pairs over the first 64
+      // columns of this group's S buffer (S is already in registers).
       float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
 #pragma unroll
-      for (int c16 = 0; c16 < 16; ++c16) {
-        float e[8];
+      for (int ch = 0; ch < 2; ++ch) {
+        float pk[32];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) e[k] = fast_exp2(fmaf(s[c16 * 8 + k], sl2, -m_use));
-        rs0 += e[0] + e[4];
-        rs1 += e[1] + e[5];
-        rs2 += e[2] + e[6];
-        rs3 += e[3] + e[7];
-        const uint32_t off = (c16 >> 3) * kHalfBytes + ((((c16 & 7) ^ (m & 7))) << 4);
-        *reinterpret_cast<uint4*>(prow + off) =
-            make_uint4(pack_bf16(e[0], e[1]), pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]),
-                       pack_bf16(e[6], e[7]));
+        for (int x = 0; x < 32; x += 2) {
+          const int c = ch * 64 + 2 * x;
+          const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
+          const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
+          const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
+          const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
+          rs0 += e0;
+          rs1 += e1;
+          rs2 += e2;
+          rs3 += e3;
+          pk[x] = __uint_as_float(pack_bf16(e0, e1));
+          pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
+        }
+        tmem_st_32x32b_x32(t_s + ch * 32, pk);
       }
       l_run += (rs0 + rs1) + (rs2 + rs3);
-      fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->p_full[grp]);
@@ -455,21 +451,25 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     const int n0 = (nt + 1) >> 1;   // tiles of group 0
     const int n1 = nt >> 1;         // tiles of group 1
     const int n_mine = grp == 0 ? n0 : n1;
-    if (n_mine > 0) {
-      if (ok) ok = wait_bar(&bars->o_done[grp], (n_mine - 1) & 1, bars, p.err);
-    }
+    // Each group waits for its own last P*V (its previous one completed before
+    // its last S, so this parity wait cannot alias an older phase); a group may
+    // own no tile when nt == 1. The barrier below then joins both groups: the
+    // last MMA of the CTA is one of the two, so every MMA has completed.
+    if (n_mine > 0 && ok) ok = wait_bar(&bars->o_done[grp], (n_mine - 1) & 1, bars, p.err);
     ok = __all_sync(0xffffffffu, ok);
+    tc_fence_before();
+    named_bar_sync(1, 256);
     tc_fence_after();
-    // Both P buffers are idle now (each group waited for its last P*V): they
-    // carry the (max, sum) exchange between the groups.
-    float* xch = reinterpret_cast<float*>(smem + kOffP + grp * kTileBytes);
+    // No Q*K^T can read Q any more: the Q buffer carries the (max, sum)
+    // exchange between the groups.
+    float* xch = reinterpret_cast<float*>(smem + kOffQ + grp * 1024);
     xch[m] = m_run;
     xch[128 + m] = l_run;
     tc_fence_before();
     named_bar_sync(1, 256);
     tc_fence_after();
-    const float* x0 = reinterpret_cast<const float*>(smem + kOffP);
-    const float* x1 = reinterpret_cast<const float*>(smem + kOffP + kTileBytes);
+    const float* x0 = reinterpret_cast<const float*>(smem + kOffQ);
+    const float* x1 = reinterpret_cast<const float*>(smem + kOffQ + 1024);
     const float mA = x0[m], lA = x0[128 + m];
     const float mB = x1[m], lB = x1[128 + m];
     const float mT = fmaxf(mA, mB);
@@ -516,12 +516,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     } else if (p.cluster) {
       // Split key range, splits of this tile in one cluster: splits > 0
       // publish their normalised partial (O_s, lse_s) in their own shared
-      // memory (the K ring, idle now) and signal split 0, which reads them
+      // memory (the K ring, idle once every Q*K^T is done) and signal split 0, which reads them
       // through distributed shared memory and merges in split order:
       //   O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M),  M = max_s lse_s.
       const float lse_own = (lT > 0.f) ? mT + __log2f(lT) : -INFINITY;
       const uint32_t xbuf = smem_u32(smem + kOffK);   // [128 rows][512 B], 16-B chunks swizzled
-      const uint32_t lbuf = smem_u32(smem + kOffV);   // [128] fp32
+      const uint32_t lbuf = smem_u32(smem + kOffK + 2 * kTileBytes);   // [128] fp32
       const uint32_t xrow = xbuf + m * 512;
       const int c_base = col0 >> 2;                  // first 16-byte chunk of my columns
       if (split > 0) {
