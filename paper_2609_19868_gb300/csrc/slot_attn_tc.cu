@@ -26,11 +26,13 @@
 //     implies P*V(i-2) is complete too. The softmax reads S with tcgen05.ld,
 //     applies the mask from indices, and runs the online softmax (exp2 on the
 //     MUFU, rescaling O only when the running maximum grows by more than 2^8);
-//   * when the key range is split across CTAs, each writes a normalised
-//     partial (O_i, log2-sum-exp_i) to the workspace and the last CTA to
-//     arrive merges them: O = sum_i 2^(lse_i - lse_max) O_i / sum_i 2^(...).
+//   * when the key range is split across CTAs, the splits of a tile form a
+//     thread-block cluster (up to 8) and merge through distributed shared
+//     memory in split order; beyond that they merge through the workspace:
+//     O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M),  M = max_s lse_s.
 //
-// Warp roles (384 threads): warp 0 K producer (and Q), warp 1 MMA issuer,
+// Warp roles (384 threads): warp 0 K producer (and Q), warp 1 MMA issuer
+// (one elected lane issues),
 // warp 2 V producer, warp 3 TMEM allocator, warps 4-7 softmax group 0 (even
 // tiles), warps 8-11 softmax group 1 (odd tiles). Warp w reads TMEM lanes
 // 32*(w%4) .. +31, i.e. the packed rows of that range.
@@ -286,58 +288,61 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
             kvh, t_begin, nt, kv_end, lane);
   } else if (warp == 1) {
-    // ======================= MMA issuer (one thread) =======================
-    if (lane == 0) {
-      bool ok = wait_bar(&bars->q_full, 0, bars, p.err);
-      bool any_mma = false;
+    // ======================= MMA issuer (one elected lane) =======================
+    // The whole warp walks the issue loop (waits and descriptors are
+    // warp-uniform); elect.sync picks the lane that issues MMAs and commits.
+    bool ok = wait_bar(&bars->q_full, 0, bars, p.err);
+    bool any_mma = false;
+    tc_fence_after();
+    const uint64_t q_desc0 = sdesc_sw128(smem_u32(smem + kOffQ), 16, 1024);
+    const uint64_t q_desc1 = sdesc_sw128(smem_u32(smem + kOffQ + kHalfBytes), 16, 1024);
+    const uint64_t k_desc0 = sdesc_sw128(smem_u32(smem + kOffK), 16, 1024);
+    const uint64_t v_desc0 = sdesc_sw128(smem_u32(smem + kOffV), kHalfBytes, 1024);
+    // descriptors count addresses in 16-byte units
+    constexpr uint64_t kTileUnits = kTileBytes >> 4, kHalfUnits = kHalfBytes >> 4;
+    auto issue_qk = [&](int i) -> bool {
+      const int s = i % kStagesK;
+      const int sb = i & 1;
+      if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
       tc_fence_after();
-      const uint32_t q_addr = smem_u32(smem + kOffQ);
-      auto issue_qk = [&](int i) -> bool {
-        const int s = i % kStagesK;
-        const int sb = i & 1;
-        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
-        tc_fence_after();
-        const uint32_t k_addr = smem_u32(smem + kOffK + s * kTileBytes);
+      const uint64_t kd = k_desc0 + s * kTileUnits;
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = sdesc_sw128(q_addr + kmajor_k_offset(kk), 16, 1024);
-          const uint64_t bd = sdesc_sw128(k_addr + kmajor_k_offset(kk), 16, 1024);
-          tc_mma_ss(tmem + sb * 128, ad, bd, kIdescQK, kk > 0 ? 1u : 0u);
-        }
-        any_mma = true;
-        tc_commit(&bars->s_full[sb]);
-        tc_commit(&bars->k_empty[s]);
-        return true;
-      };
-      auto issue_pv = [&](int i) -> bool {
-        const int sv = i % kStagesV;
-        const int sb = i & 1;
-        const int j = i >> 1;
-        if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
-        if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(smem + kOffV + sv * kTileBytes);
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t step = (kk >> 2) * kHalfUnits + (kk & 3) * 2;
+        tc_mma_ss_elect(tmem + sb * 128, (kk < 4 ? q_desc0 : q_desc1) + (kk & 3) * 2,
+                        kd + step, kIdescQK, kk > 0 ? 1u : 0u);
+      }
+      any_mma = true;
+      tc_commit_elect(&bars->s_full[sb]);
+      tc_commit_elect(&bars->k_empty[s]);
+      return true;
+    };
+    auto issue_pv = [&](int i) -> bool {
+      const int sv = i % kStagesV;
+      const int sb = i & 1;
+      const int j = i >> 1;
+      if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
+      if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
+      tc_fence_after();
+      const uint64_t vd = v_desc0 + sv * kTileUnits;
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t bd = sdesc_sw128(v_addr + kk * 2048, kHalfBytes, 1024);
-          tc_mma_ts(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, bd, kIdescPV,
-                    (j > 0 || kk > 0) ? 1u : 0u);
-        }
-        any_mma = true;
-        tc_commit(&bars->o_done[sb]);
-        tc_commit(&bars->v_empty[sv]);
-        return true;
-      };
-      if (ok) ok = issue_qk(0);
-      if (ok && nt > 1) ok = issue_qk(1);
-      for (int i = 0; i < nt && ok; ++i) {
-        if (!issue_pv(i)) { ok = false; break; }
-        if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
-      }
-      if (!ok && any_mma) {
-        tc_commit(&bars->drain);
-        mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
-      }
+      for (int kk = 0; kk < 8; ++kk)
+        tc_mma_ts_elect(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, vd + kk * 128,
+                        kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+      any_mma = true;
+      tc_commit_elect(&bars->o_done[sb]);
+      tc_commit_elect(&bars->v_empty[sv]);
+      return true;
+    };
+    if (ok) ok = issue_qk(0);
+    if (ok && nt > 1) ok = issue_qk(1);
+    for (int i = 0; i < nt && ok; ++i) {
+      if (!issue_pv(i)) { ok = false; break; }
+      if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
+    }
+    if (!ok && any_mma) {
+      tc_commit_elect(&bars->drain);
+      mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
     }
   } else if (warp >= 4) {
     // ======================= softmax + epilogue =======================
@@ -418,6 +423,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
             reinterpret_cast<uint4*>(vrow + kHalfBytes)[x] = z;
           }
         }
+        // the zeros are generic-proxy writes; P*V reads V through the async proxy
+        fence_proxy_async_smem();
       }
       // P = 2^(s * scale * log2 e - m) as packed bf16 pairs over the first 64
       // columns of this group's S buffer (S is already in registers).
