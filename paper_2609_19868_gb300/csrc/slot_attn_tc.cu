@@ -27,8 +27,9 @@
 //     applies the mask from indices, and runs the online softmax (exp2 on the
 //     MUFU, rescaling O only when the running maximum grows by more than 2^8);
 //   * when the key range is split across CTAs, the splits of a tile form a
-//     thread-block cluster (up to 8) and merge through distributed shared
-//     memory in split order; beyond that they merge through the workspace:
+//     thread-block cluster (up to 3): splits > 0 push their partial into
+//     split 0's shared memory with a bulk copy and split 0 merges in split
+//     order; more splits merge through the workspace:
 //     O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M),  M = max_s lse_s.
 //
 // Warp roles (384 threads): warp 0 K producer (and Q), warp 1 MMA issuer
@@ -73,8 +74,8 @@ struct Bars {
   uint64_t p_full[2];
   uint64_t o_done[2];
   uint64_t drain;
-  uint64_t ready;   // split 0: the other splits' partials are published
-  uint64_t done;    // splits > 0: split 0 has read this CTA's partial
+  uint64_t ready;   // split 0: the other splits' partials have landed (tx bytes)
+  uint64_t go;      // splits > 0: split 0's K/V rings are free to receive
   uint32_t tmem_base;
   int abort;
   int last;
@@ -244,8 +245,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       mbar_init(&bars->o_done[s], 1);
     }
     mbar_init(&bars->drain, 1);
-    mbar_init(&bars->ready, active > 1 ? active - 1 : 1);
-    mbar_init(&bars->done, 1);
+    mbar_init(&bars->ready, 1);
+    mbar_init(&bars->go, 1);
     bars->abort = 0;
     bars->last = 0;
     fence_mbar_init();
@@ -521,17 +522,26 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     if (active == 1) {
       if (ok && row_ok) store_out(o, 1.f);
     } else if (p.cluster) {
-      // Split key range, splits of this tile in one cluster: splits > 0
-      // publish their normalised partial (O_s, lse_s) in their own shared
-      // memory (the K ring, idle once every Q*K^T is done) and signal split 0, which reads them
-      // through distributed shared memory and merges in split order:
-      //   O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M),  M = max_s lse_s.
+      // Split key range, splits of this tile in one cluster (at most 3). Once
+      // split 0 has finished its loop its K and V rings are idle: it arms its
+      // `ready` barrier for the bytes to come and tells the other splits to
+      // go. Each pushes its normalised partial (valid rows of O_s, lse_s) from
+      // its own shared memory into split 0's rings with one bulk copy per
+      // array; split 0 then merges from local shared memory in split order:
+      //   O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M).
       const float lse_own = (lT > 0.f) ? mT + __log2f(lT) : -INFINITY;
-      const uint32_t xbuf = smem_u32(smem + kOffK);   // [128 rows][512 B], 16-B chunks swizzled
-      const uint32_t lbuf = smem_u32(smem + kOffK + 2 * kTileBytes);   // [128] fp32
-      const uint32_t xrow = xbuf + m * 512;
+      const int n_rows = min(kBlockM, (r_hi - r0 + 1) * p.g);   // valid packed rows
+      const uint32_t row_bytes = static_cast<uint32_t>(n_rows) * 512u;
+      const uint32_t lse_bytes = (static_cast<uint32_t>(n_rows) * 4u + 15u) & ~15u;
       const int c_base = col0 >> 2;                  // first 16-byte chunk of my columns
+      // partial s lives at region(s): s = 1 in the K ring, s = 2 in the V ring
+      auto region = [&](int sp) -> uint32_t {
+        return smem_u32(smem + (sp == 1 ? kOffK : kOffV));
+      };
       if (split > 0) {
+        const uint32_t xbuf = smem_u32(smem + kOffK);        // own rows, same layout
+        const uint32_t lbuf = xbuf + 64 * 1024;
+        const uint32_t xrow = xbuf + m * 512;
         if (ok && row_ok) {
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
@@ -543,33 +553,39 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           if (grp == 0)
             asm volatile("st.shared.f32 [%0], %1;" ::"r"(lbuf + m * 4), "f"(lse_own) : "memory");
         }
+        fence_proxy_async_smem();   // the bulk copy reads through the async proxy
         named_bar_sync(1, 256);
-        if (grp == 0 && m == 0) {
-          if (*reinterpret_cast<volatile int*>(&bars->abort) == 0) {
-            mbar_arrive_remote(mapa_shared(smem_u32(&bars->ready), 0));
-            // split 0 reads this CTA's shared memory: stay until it is done
-            if (!mbar_wait_cluster(&bars->done, 0, kWaitNs, nullptr))
-              set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
+        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->abort) == 0) {
+          if (mbar_wait_cluster(&bars->go, 0, kWaitNs, nullptr)) {
+            const uint32_t dst = mapa_shared(region(split), 0);
+            const uint32_t rbar = mapa_shared(smem_u32(&bars->ready), 0);
+            bulk_copy_to_cluster(dst, xbuf, row_bytes, rbar);
+            bulk_copy_to_cluster(dst + 64 * 1024, lbuf, lse_bytes, rbar);
+            bulk_commit_and_wait_read();   // this CTA's smem must outlive the reads
+          } else {
+            set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
           }
         }
         named_bar_sync(1, 256);
       } else {
-        if (grp == 0 && m == 0) {
-          const bool got = mbar_wait_cluster(&bars->ready, 0, kWaitNs, &bars->abort);
-          if (!got) set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
-          bars->last = got ? 1 : 0;
+        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->abort) == 0) {
+          mbar_arrive_expect_tx(&bars->ready, (active - 1) * (row_bytes + lse_bytes));
+          for (int sp = 1; sp < active; ++sp)
+            mbar_arrive_remote(mapa_shared(smem_u32(&bars->go), sp));
         }
-        named_bar_sync(1, 256);
-        if (*reinterpret_cast<volatile int*>(&bars->last) && ok && row_ok) {
+        // every reader observes the bulk copies' completion itself
+        const bool got = __all_sync(0xffffffffu, wait_bar(&bars->ready, 0, bars, p.err));
+        if (got && ok && row_ok) {
           float M = lse_own;
           float S = (lse_own == -INFINITY) ? 0.f : 1.f;
           for (int sp = 1; sp < active; ++sp) {
-            const float ls = ld_shared_cluster_f32(mapa_shared(lbuf + m * 4, sp));
-            const uint32_t rx = mapa_shared(xrow, sp);
+            const uint8_t* rbase = smem + (sp == 1 ? kOffK : kOffV);
+            const float ls = reinterpret_cast<const float*>(rbase + 64 * 1024)[m];
+            const uint8_t* rrow = rbase + m * 512;
             float4 v[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c)
-              v[c] = ld_shared_cluster_f4(rx + ((((c_base + c) ^ (m & 31))) << 4));
+              v[c] = *reinterpret_cast<const float4*>(rrow + ((((c_base + c) ^ (m & 31))) << 4));
             const float Mn = fmaxf(M, ls);
             const float a = (M == -INFINITY) ? 0.f : fast_exp2(M - Mn);
             const float c2 = (ls == -INFINITY) ? 0.f : fast_exp2(ls - Mn);
@@ -585,10 +601,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           }
           store_out(o, S > 0.f ? 1.f / S : 0.f);
         }
-        named_bar_sync(1, 256);
-        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->last))
-          for (int sp = 1; sp < active; ++sp)
-            mbar_arrive_remote(mapa_shared(smem_u32(&bars->done), sp));
       }
     } else {
       // Split key range beyond a cluster: every split writes its partial to

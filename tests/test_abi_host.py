@@ -106,8 +106,8 @@ def test_workspace_size_for_forced_splits(lib):
     expect = (expect + 255) // 256 * 256 + 16 * 4
     expect = (expect + 255) // 256 * 256
     assert lib.zarya_slot_attn_workspace_size(ctypes.byref(d)) == expect
-    # up to 8 splits merge inside a cluster and need no workspace
-    for s in (1, 2, 8):
+    # up to 3 splits merge inside a thread-block cluster and need no workspace
+    for s in (1, 2, 3):
         d = _desc(kv_splits=s, cache_capacity=2048)
         assert lib.zarya_slot_attn_workspace_size(ctypes.byref(d)) == 0
 
