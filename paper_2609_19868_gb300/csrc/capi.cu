@@ -83,7 +83,6 @@ zarya_status check_attn_support(const zarya_attn_desc* d) {
   return ZARYA_OK;
 }
 
-constexpr int kMaxClusterSplits = 3;  // split 0 receives two partials in its K/V rings
 
 struct Plan {
   int g, m_tiles, splits;

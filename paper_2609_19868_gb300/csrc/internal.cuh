@@ -14,6 +14,9 @@ namespace zarya {
 constexpr int kBlockM = 128;  // packed (block row, query head) rows per CTA
 constexpr int kBlockN = 128;  // keys per pipeline tile
 constexpr int kHeadDim = 128;
+// At most this many key splits of one tile merge inside a thread-block cluster
+// (each split receives the rows it finishes from the others in its idle K ring).
+constexpr int kMaxClusterSplits = 3;
 
 // Parameters of the tensor-core slot-attention kernel (tensor maps travel as
 // separate __grid_constant__ arguments).

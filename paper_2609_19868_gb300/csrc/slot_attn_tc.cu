@@ -61,6 +61,11 @@ constexpr uint32_t kOffV = kOffK + kStagesK * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStagesV * kTileBytes;
 constexpr uint32_t kTmemCols = 512;  // S0/P0 [0,128) S1/P1 [128,256) O0 [256,384) O1 [384,512)
 constexpr uint32_t kTmemO = 256;
+constexpr int kRegsLaunch = 168;    // 65536 / 384, rounded down to a multiple of 8
+constexpr int kRegsControl = 64;    // warps 0-3
+constexpr int kRegsSoftmax = 216;   // warps 4-11
+static_assert(4 * 32 * kRegsControl + 8 * 32 * kRegsSoftmax <= kThreads * kRegsLaunch,
+              "register split exceeds the launch allocation");
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
 constexpr uint64_t kDrainNs = 100000000ull;  // 100 ms
 
@@ -74,8 +79,9 @@ struct Bars {
   uint64_t p_full[2];
   uint64_t o_done[2];
   uint64_t drain;
-  uint64_t ready;   // split 0: the other splits' partials have landed (tx bytes)
-  uint64_t go;      // splits > 0: split 0's K/V rings are free to receive
+  uint64_t kfree;   // this CTA's last Q*K^T has completed: its K ring is idle
+  uint64_t ready;   // cluster merge: every partial row this CTA owns has landed
+  uint64_t go;      // cluster merge: every other split's K ring is free to receive
   uint32_t tmem_base;
   int abort;
   int last;
@@ -113,10 +119,111 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Bars* b
   return false;
 }
 
-// Offset (bytes) of the k-th 16-element K slice inside a 128-row, 2-half,
-// K-major SW128 tile.
-__device__ __forceinline__ uint32_t kmajor_k_offset(int kk) {
-  return (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+// Cluster merge layout. Packed rows are handled in quadrants of 32 (one warp
+// of each softmax group); quadrant q is finished by split q % active. A
+// quadrant's partial (32 rows x 128 fp32 columns, 16 KB, plus 32 lse values)
+// is staged by each other split in its idle V ring and pushed with one bulk
+// copy into the owner's idle K ring, slot (sender's rank among the owner's
+// peers, q / active).
+constexpr uint32_t kQuadBytes = 32 * kHeadDim * 4;
+constexpr uint32_t kQuadLseBytes = 32 * 4;
+constexpr uint32_t kRxLse = 64 * 1024;   // lse slots follow the data slots
+
+__device__ __forceinline__ uint32_t cmerge_rx_bytes(int n_rows, int active, int split) {
+  const int nq = (n_rows + 31) >> 5;
+  int owned = 0;
+  for (int q = split; q < nq; q += active) ++owned;
+  return static_cast<uint32_t>((active - 1) * owned) * (kQuadBytes + kQuadLseBytes);
+}
+
+// Swizzled byte offset of 16-byte chunk `chunk` (0..31) of row `L` (0..31) of
+// a quadrant: lanes L of a warp touch distinct chunks of their rows.
+__device__ __forceinline__ uint32_t quad_chunk(int L, int chunk) {
+  return static_cast<uint32_t>(L) * 512u + (static_cast<uint32_t>(chunk ^ L) << 4);
+}
+
+__device__ __forceinline__ void st_shared_f4(uint32_t a, float x, float y, float z, float w) {
+  asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(x), "f"(y), "f"(z),
+               "f"(w)
+               : "memory");
+}
+
+__device__ __forceinline__ float4 ld_shared_f4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(a)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float ld_shared_f32(uint32_t a) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+
+// Owner side of the cluster merge for one row: this split's normalised
+// partial o (64 columns of group grp) and the A - 1 partials received from the
+// other splits, O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M), stored as
+// bf16. rx / rx_lse address the first peer slot of this row (shared::cta).
+template <int A>
+__device__ __forceinline__ void cluster_merge_store(const float (&o)[64], float lse_own,
+                                                    uint32_t rx, uint32_t rx_lse, int L, int grp,
+                                                    __nv_bfloat16* out_row) {
+  float lp[A - 1];
+  float M = lse_own;
+#pragma unroll
+  for (int k = 0; k < A - 1; ++k) {
+    lp[k] = ld_shared_f32(rx_lse + k * 2 * kQuadLseBytes);
+    M = fmaxf(M, lp[k]);
+  }
+  float wo = lse_own == -INFINITY ? 0.f : fast_exp2(lse_own - M);
+  float wp[A - 1];
+  float S = wo;
+#pragma unroll
+  for (int k = 0; k < A - 1; ++k) {
+    wp[k] = lp[k] == -INFINITY ? 0.f : fast_exp2(lp[k] - M);
+    S += wp[k];
+  }
+  const float inv = S > 0.f ? 1.f / S : 0.f;
+  wo *= inv;
+#pragma unroll
+  for (int k = 0; k < A - 1; ++k) wp[k] *= inv;
+  uint4* d4 = reinterpret_cast<uint4*>(out_row);
+#pragma unroll
+  for (int x = 0; x < 8; ++x) {
+    float r[8];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = 2 * x + h;
+      float4 acc = make_float4(wo * o[4 * c], wo * o[4 * c + 1], wo * o[4 * c + 2], wo * o[4 * c + 3]);
+#pragma unroll
+      for (int k = 0; k < A - 1; ++k) {
+        const float4 v = ld_shared_f4(rx + k * 2 * kQuadBytes + quad_chunk(L, grp * 16 + c) -
+                                      static_cast<uint32_t>(L) * 512u);
+        acc.x = fmaf(wp[k], v.x, acc.x);
+        acc.y = fmaf(wp[k], v.y, acc.y);
+        acc.z = fmaf(wp[k], v.z, acc.z);
+        acc.w = fmaf(wp[k], v.w, acc.w);
+      }
+      r[4 * h] = acc.x;
+      r[4 * h + 1] = acc.y;
+      r[4 * h + 2] = acc.z;
+      r[4 * h + 3] = acc.w;
+    }
+    d4[x] = make_uint4(pack_bf16(r[0], r[1]), pack_bf16(r[2], r[3]), pack_bf16(r[4], r[5]),
+                       pack_bf16(r[6], r[7]));
+  }
+}
+
+// Bounded wait (acquire at cluster scope) for a phase completed by other CTAs
+// of the cluster.
+__device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity, Bars* bars,
+                                                 int* err) {
+  if (mbar_wait_cluster(bar, parity, kWaitNs, &bars->abort)) return true;
+  set_abort(bars, err, ZARYA_DEVERR_TIMEOUT);
+  return false;
 }
 
 // One producer warp streams one of K or V through its ring.
@@ -205,6 +312,26 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     tma_prefetch_map(&map_k);
     tma_prefetch_map(&map_v);
   }
+  if (threadIdx.x == 32) {
+    mbar_init(&bars->q_full, 1);
+    for (int s = 0; s < kStagesK; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+    }
+    for (int s = 0; s < kStagesV; ++s) {
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars->s_full[s], 1);
+      mbar_init(&bars->p_full[s], 4);
+      mbar_init(&bars->o_done[s], 1);
+    }
+    mbar_init(&bars->drain, 1);
+    mbar_init(&bars->kfree, 1);
+    bars->abort = 0;
+    bars->last = 0;
+  }
   // Inputs may be written by the kernel launched before this one.
   grid_dependency_wait();
 
@@ -229,123 +356,132 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   const int t_begin = split * per_split;
   const int nt = min(n_tiles, t_begin + per_split) - t_begin;
 
-  if (threadIdx.x == 0) {
-    mbar_init(&bars->q_full, 1);
-    for (int s = 0; s < kStagesK; ++s) {
-      mbar_init(&bars->k_full[s], 1);
-      mbar_init(&bars->k_empty[s], 1);
-    }
-    for (int s = 0; s < kStagesV; ++s) {
-      mbar_init(&bars->v_full[s], 1);
-      mbar_init(&bars->v_empty[s], 1);
-    }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&bars->s_full[s], 1);
-      mbar_init(&bars->p_full[s], 4);
-      mbar_init(&bars->o_done[s], 1);
-    }
-    mbar_init(&bars->drain, 1);
+  // The splits of a cluster merge their partials through shared memory when
+  // more than one of them has keys (Sec. 5.2 step 3 split over the key range).
+  const bool cmerge = p.cluster != 0 && active > 1;
+  if (threadIdx.x == 32) {
+    mbar_init(&bars->go, cmerge ? active - 1 : 1);
     mbar_init(&bars->ready, 1);
-    mbar_init(&bars->go, 1);
-    bars->abort = 0;
-    bars->last = 0;
     fence_mbar_init();
+    // The bytes the other splits will push (their rows of the quadrants this
+    // split finishes) are known here, so the barrier is armed before any peer
+    // can start a copy.
+    if (cmerge) {
+      const int n_rows_v = min(kBlockM, (r_hi - r0 + 1) * p.g);
+      mbar_arrive_expect_tx(&bars->ready, cmerge_rx_bytes(n_rows_v, active, split));
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
-  // Exits before the cluster barrier are uniform over a cluster (its CTAs
-  // share the sequence and M-tile and differ only in the split).
-  if (code != 0 || r0 >= R) {
+  // The cluster barrier orders every CTA's barrier initialisation before any
+  // remote arrive; its wait is taken only where a thread first needs it.
+  if (p.cluster) cluster_arrive();
+  bool cwaited = false;
+  // Exits here are uniform over a cluster (its CTAs share the sequence and
+  // M-tile and differ only in the split) or leave a split with no keys.
+  if (code != 0 || r0 >= R || split >= active) {
     if (code != 0 && mt == 0 && split == 0 && threadIdx.x == 0) record_error(p.err, code);
     grid_launch_dependents();
-    if (warp == 3) tmem_dealloc(tmem, kTmemCols);
-    return;
-  }
-  // Every CTA of the cluster has initialised its barriers before any remote
-  // arrive can target them.
-  if (p.cluster) cluster_sync();
-  if (split >= active) {
-    grid_launch_dependents();
+    if (p.cluster) cluster_wait();
     if (warp == 3) tmem_dealloc(tmem, kTmemCols);
     return;
   }
 
-  if (warp == 0) {
-    // ======================= Q + K producer =======================
-    if (lane == 0) {
-      mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
-      const uint32_t dq = smem_u32(smem + kOffQ);
-      tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
-      tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
-    }
-    produce(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars, b,
-            kvh, t_begin, nt, kv_end, lane);
-    if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
-      mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
-  } else if (warp == 2) {
-    // ======================= V producer =======================
-    produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
-            kvh, t_begin, nt, kv_end, lane);
-  } else if (warp == 1) {
-    // ======================= MMA issuer (one elected lane) =======================
-    // The whole warp walks the issue loop (waits and descriptors are
-    // warp-uniform); elect.sync picks the lane that issues MMAs and commits.
-    bool ok = wait_bar(&bars->q_full, 0, bars, p.err);
-    bool any_mma = false;
-    tc_fence_after();
-    const uint64_t q_desc0 = sdesc_sw128(smem_u32(smem + kOffQ), 16, 1024);
-    const uint64_t q_desc1 = sdesc_sw128(smem_u32(smem + kOffQ + kHalfBytes), 16, 1024);
-    const uint64_t k_desc0 = sdesc_sw128(smem_u32(smem + kOffK), 16, 1024);
-    const uint64_t v_desc0 = sdesc_sw128(smem_u32(smem + kOffV), kHalfBytes, 1024);
-    // descriptors count addresses in 16-byte units
-    constexpr uint64_t kTileUnits = kTileBytes >> 4, kHalfUnits = kHalfBytes >> 4;
-    auto issue_qk = [&](int i) -> bool {
-      const int s = i % kStagesK;
-      const int sb = i & 1;
-      if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
-      tc_fence_after();
-      const uint64_t kd = k_desc0 + s * kTileUnits;
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t step = (kk >> 2) * kHalfUnits + (kk & 3) * 2;
-        tc_mma_ss_elect(tmem + sb * 128, (kk < 4 ? q_desc0 : q_desc1) + (kk & 3) * 2,
-                        kd + step, kIdescQK, kk > 0 ? 1u : 0u);
+  // Registers: the producer / MMA / TMEM warpgroup hands most of its share to
+  // the two softmax warpgroups (128 x 64 + 256 x 216 <= 384 x 168 at launch).
+  if (warp < 4) {
+    regs_release<kRegsControl>();
+    if (warp == 0) {
+      // ======================= Q + K producer =======================
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
+        const uint32_t dq = smem_u32(smem + kOffQ);
+        tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
+        tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
       }
-      any_mma = true;
-      tc_commit_elect(&bars->s_full[sb]);
-      tc_commit_elect(&bars->k_empty[s]);
-      return true;
-    };
-    auto issue_pv = [&](int i) -> bool {
-      const int sv = i % kStagesV;
-      const int sb = i & 1;
-      const int j = i >> 1;
-      if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
-      if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
+      produce(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars, b,
+              kvh, t_begin, nt, kv_end, lane);
+      if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
+        mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
+    } else if (warp == 2) {
+      // ======================= V producer =======================
+      produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
+              kvh, t_begin, nt, kv_end, lane);
+    } else if (warp == 1) {
+      // ======================= MMA issuer (one elected lane) =======================
+      // The whole warp walks the issue loop (waits and descriptors are
+      // warp-uniform); elect.sync picks the lane that issues MMAs and commits.
+      bool ok = wait_bar(&bars->q_full, 0, bars, p.err);
+      bool any_mma = false;
       tc_fence_after();
-      const uint64_t vd = v_desc0 + sv * kTileUnits;
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk)
-        tc_mma_ts_elect(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, vd + kk * 128,
-                        kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
-      any_mma = true;
-      tc_commit_elect(&bars->o_done[sb]);
-      tc_commit_elect(&bars->v_empty[sv]);
-      return true;
-    };
-    if (ok) ok = issue_qk(0);
-    if (ok && nt > 1) ok = issue_qk(1);
-    for (int i = 0; i < nt && ok; ++i) {
-      if (!issue_pv(i)) { ok = false; break; }
-      if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
+      const uint64_t q_desc0 = sdesc_sw128(smem_u32(smem + kOffQ), 16, 1024);
+      const uint64_t q_desc1 = sdesc_sw128(smem_u32(smem + kOffQ + kHalfBytes), 16, 1024);
+      const uint64_t k_desc0 = sdesc_sw128(smem_u32(smem + kOffK), 16, 1024);
+      const uint64_t v_desc0 = sdesc_sw128(smem_u32(smem + kOffV), kHalfBytes, 1024);
+      // descriptors count addresses in 16-byte units
+      constexpr uint64_t kTileUnits = kTileBytes >> 4, kHalfUnits = kHalfBytes >> 4;
+      auto issue_qk = [&](int i) -> bool {
+        const int s = i % kStagesK;
+        const int sb = i & 1;
+        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
+        tc_fence_after();
+        const uint64_t kd = k_desc0 + s * kTileUnits;
+  #pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t step = (kk >> 2) * kHalfUnits + (kk & 3) * 2;
+          tc_mma_ss_elect(tmem + sb * 128, (kk < 4 ? q_desc0 : q_desc1) + (kk & 3) * 2,
+                          kd + step, kIdescQK, kk > 0 ? 1u : 0u);
+        }
+        any_mma = true;
+        tc_commit_elect(&bars->s_full[sb]);
+        tc_commit_elect(&bars->k_empty[s]);
+        if (cmerge && i == nt - 1) tc_commit_elect(&bars->kfree);
+        return true;
+      };
+      auto issue_pv = [&](int i) -> bool {
+        const int sv = i % kStagesV;
+        const int sb = i & 1;
+        const int j = i >> 1;
+        if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
+        if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
+        tc_fence_after();
+        const uint64_t vd = v_desc0 + sv * kTileUnits;
+  #pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          tc_mma_ts_elect(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, vd + kk * 128,
+                          kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+        any_mma = true;
+        tc_commit_elect(&bars->o_done[sb]);
+        tc_commit_elect(&bars->v_empty[sv]);
+        return true;
+      };
+      if (ok) ok = issue_qk(0);
+      if (ok && nt > 1) ok = issue_qk(1);
+      for (int i = 0; i < nt && ok; ++i) {
+        if (!issue_pv(i)) { ok = false; break; }
+        if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
+      }
+      if (!ok && any_mma) {
+        tc_commit_elect(&bars->drain);
+        mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
+      }
+    } else if (warp == 3) {
+      // ======================= cluster merge: K ring hand-off =======================
+      // Once this CTA's last Q*K^T has completed no copy or MMA touches its K
+      // ring again: tell the other splits they may write their rows into it.
+      if (cmerge) {
+        const bool freed = wait_bar(&bars->kfree, 0, bars, p.err);
+        cluster_wait();
+        cwaited = true;
+        if (freed && lane == 0)
+          for (int sp = 0; sp < active; ++sp)
+            if (sp != split) mbar_arrive_remote(mapa_shared(smem_u32(&bars->go), sp));
+      }
     }
-    if (!ok && any_mma) {
-      tc_commit_elect(&bars->drain);
-      mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
-    }
-  } else if (warp >= 4) {
+  } else {
+    regs_claim<kRegsSoftmax>();
     // ======================= softmax + epilogue =======================
     const int grp = (warp - 4) >> 2;                // 0: even tiles, 1: odd tiles
     const int wq = warp & 3;
@@ -522,84 +658,53 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     if (active == 1) {
       if (ok && row_ok) store_out(o, 1.f);
     } else if (p.cluster) {
-      // Split key range, splits of this tile in one cluster (at most 3). Once
-      // split 0 has finished its loop its K and V rings are idle: it arms its
-      // `ready` barrier for the bytes to come and tells the other splits to
-      // go. Each pushes its normalised partial (valid rows of O_s, lse_s) from
-      // its own shared memory into split 0's rings with one bulk copy per
-      // array; split 0 then merges from local shared memory in split order:
+      // Split key range, the splits of this tile in one cluster (at most 3).
+      // Each quadrant of 32 packed rows is finished by split q % active; the
+      // other splits stage their normalised partial of it (O_s, lse_s) in
+      // their idle V ring and, once the owner's K ring is idle (its `go`),
+      // push it there with one bulk copy that completes on the owner's
+      // `ready`. The owner merges
       //   O = sum_s 2^(lse_s - M) O_s / sum_s 2^(lse_s - M).
       const float lse_own = (lT > 0.f) ? mT + __log2f(lT) : -INFINITY;
       const int n_rows = min(kBlockM, (r_hi - r0 + 1) * p.g);   // valid packed rows
-      const uint32_t row_bytes = static_cast<uint32_t>(n_rows) * 512u;
-      const uint32_t lse_bytes = (static_cast<uint32_t>(n_rows) * 4u + 15u) & ~15u;
-      const int c_base = col0 >> 2;                  // first 16-byte chunk of my columns
-      // partial s lives at region(s): s = 1 in the K ring, s = 2 in the V ring
-      auto region = [&](int sp) -> uint32_t {
-        return smem_u32(smem + (sp == 1 ? kOffK : kOffV));
-      };
-      if (split > 0) {
-        const uint32_t xbuf = smem_u32(smem + kOffK);        // own rows, same layout
-        const uint32_t lbuf = xbuf + 64 * 1024;
-        const uint32_t xrow = xbuf + m * 512;
-        if (ok && row_ok) {
+      const int q = wq;                                          // this warp's quadrant
+      const int owner = q % active;
+      const uint32_t sbase = smem_u32(smem);
+      cluster_wait();
+      cwaited = true;
+      if (q * 32 < n_rows && owner != split) {
+        const uint32_t stage = sbase + kOffV + q * kQuadBytes;
+        const uint32_t stage_lse = sbase + kOffV + kRxLse + q * kQuadLseBytes;
 #pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const uint32_t a = xrow + ((((c_base + c) ^ (m & 31))) << 4);
-            asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(o[4 * c]),
-                         "f"(o[4 * c + 1]), "f"(o[4 * c + 2]), "f"(o[4 * c + 3])
-                         : "memory");
-          }
-          if (grp == 0)
-            asm volatile("st.shared.f32 [%0], %1;" ::"r"(lbuf + m * 4), "f"(lse_own) : "memory");
-        }
+        for (int c = 0; c < 16; ++c)
+          st_shared_f4(stage + quad_chunk(lane, grp * 16 + c), o[4 * c], o[4 * c + 1], o[4 * c + 2],
+                       o[4 * c + 3]);
+        if (grp == 0)
+          asm volatile("st.shared.f32 [%0], %1;" ::"r"(stage_lse + lane * 4), "f"(lse_own)
+                       : "memory");
         fence_proxy_async_smem();   // the bulk copy reads through the async proxy
-        named_bar_sync(1, 256);
-        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->abort) == 0) {
-          if (mbar_wait_cluster(&bars->go, 0, kWaitNs, nullptr)) {
-            const uint32_t dst = mapa_shared(region(split), 0);
-            const uint32_t rbar = mapa_shared(smem_u32(&bars->ready), 0);
-            bulk_copy_to_cluster(dst, xbuf, row_bytes, rbar);
-            bulk_copy_to_cluster(dst + 64 * 1024, lbuf, lse_bytes, rbar);
+        named_bar_sync(2 + q, 64);  // this quadrant's warp of each group
+        if (grp == 0 && lane == 0) {
+          if (wait_bar_cluster(&bars->go, 0, bars, p.err)) {
+            const int slot = (split < owner ? split : split - 1) * 2 + q / active;
+            const uint32_t rbar = mapa_shared(smem_u32(&bars->ready), owner);
+            bulk_copy_to_cluster(mapa_shared(sbase + kOffK + slot * kQuadBytes, owner), stage,
+                                 kQuadBytes, rbar);
+            bulk_copy_to_cluster(mapa_shared(sbase + kOffK + kRxLse + slot * kQuadLseBytes, owner),
+                                 stage_lse, kQuadLseBytes, rbar);
             bulk_commit_and_wait_read();   // this CTA's smem must outlive the reads
-          } else {
-            set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
           }
         }
-        named_bar_sync(1, 256);
-      } else {
-        if (grp == 0 && m == 0 && *reinterpret_cast<volatile int*>(&bars->abort) == 0) {
-          mbar_arrive_expect_tx(&bars->ready, (active - 1) * (row_bytes + lse_bytes));
-          for (int sp = 1; sp < active; ++sp)
-            mbar_arrive_remote(mapa_shared(smem_u32(&bars->go), sp));
-        }
-        // every reader observes the bulk copies' completion itself
-        const bool got = __all_sync(0xffffffffu, wait_bar(&bars->ready, 0, bars, p.err));
+      } else if (q * 32 < n_rows) {
+        const bool got = wait_bar_cluster(&bars->ready, 0, bars, p.err);
         if (got && ok && row_ok) {
-          float M = lse_own;
-          float S = (lse_own == -INFINITY) ? 0.f : 1.f;
-          for (int sp = 1; sp < active; ++sp) {
-            const uint8_t* rbase = smem + (sp == 1 ? kOffK : kOffV);
-            const float ls = reinterpret_cast<const float*>(rbase + 64 * 1024)[m];
-            const uint8_t* rrow = rbase + m * 512;
-            float4 v[16];
-#pragma unroll
-            for (int c = 0; c < 16; ++c)
-              v[c] = *reinterpret_cast<const float4*>(rrow + ((((c_base + c) ^ (m & 31))) << 4));
-            const float Mn = fmaxf(M, ls);
-            const float a = (M == -INFINITY) ? 0.f : fast_exp2(M - Mn);
-            const float c2 = (ls == -INFINITY) ? 0.f : fast_exp2(ls - Mn);
-            S = S * a + c2;
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-              o[4 * c + 0] = o[4 * c + 0] * a + c2 * v[c].x;
-              o[4 * c + 1] = o[4 * c + 1] * a + c2 * v[c].y;
-              o[4 * c + 2] = o[4 * c + 2] * a + c2 * v[c].z;
-              o[4 * c + 3] = o[4 * c + 3] * a + c2 * v[c].w;
-            }
-            M = Mn;
-          }
-          store_out(o, S > 0.f ? 1.f / S : 0.f);
+          const int j = q / active;
+          const uint32_t rx = sbase + kOffK + j * kQuadBytes + lane * 512u;
+          const uint32_t rx_lse = sbase + kOffK + kRxLse + j * kQuadLseBytes + lane * 4u;
+          if (active == 2)
+            cluster_merge_store<2>(o, lse_own, rx, rx_lse, lane, grp, out_row);
+          else
+            cluster_merge_store<3>(o, lse_own, rx, rx_lse, lane, grp, out_row);
         }
       }
     } else {
@@ -659,6 +764,10 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   }
 
   // ---- teardown ----
+  if (p.cluster && !cwaited) cluster_wait();
+  // Every other split's `go` arrive has landed before this CTA's shared
+  // memory goes away.
+  if (cmerge && threadIdx.x == 0) wait_bar_cluster(&bars->go, 0, bars, p.err);
   tc_fence_before();
   __syncthreads();
   if (warp == 3) {
