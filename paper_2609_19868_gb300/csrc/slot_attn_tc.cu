@@ -77,7 +77,7 @@ struct Bars {
   uint64_t v_empty[kStagesV];
   uint64_t s_full[2];
   uint64_t p_full[2];
-  uint64_t o_done[2];
+  uint64_t o_done[2];   // o_done[i & 1], phase i >> 1: P*V(i) has completed
   uint64_t drain;
   uint64_t kfree;   // this CTA's last Q*K^T has completed: its K ring is idle
   uint64_t ready;   // cluster merge: every partial row this CTA owns has landed
@@ -324,9 +324,10 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bars->s_full[s], 1);
-      mbar_init(&bars->p_full[s], 4);
-      mbar_init(&bars->o_done[s], 1);
+      mbar_init(&bars->p_full[s], 8);   // every softmax warp, each tile
     }
+    mbar_init(&bars->o_done[0], 1);
+    mbar_init(&bars->o_done[1], 1);
     mbar_init(&bars->drain, 1);
     mbar_init(&bars->kfree, 1);
     bars->abort = 0;
@@ -448,10 +449,14 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
         tc_fence_after();
         const uint64_t vd = v_desc0 + sv * kTileUnits;
+        // O_g += P_g(i) * V(i)[64g, 64g + 64): P_g is packed over columns
+        // [64g, 64g + 32) of the tile's S buffer, 16 keys per 8 columns.
   #pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          tc_mma_ts_elect(tmem + kTmemO + sb * 128, tmem + sb * 128 + kk * 8, vd + kk * 128,
-                          kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+        for (int g2 = 0; g2 < 2; ++g2)
+  #pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_ts_elect(tmem + kTmemO + g2 * 128, tmem + sb * 128 + g2 * 64 + kk * 8,
+                            vd + (g2 * 4 + kk) * 128, kIdescPV, (i > 0 || kk > 0) ? 1u : 0u);
         any_mma = true;
         tc_commit_elect(&bars->o_done[sb]);
         tc_commit_elect(&bars->v_empty[sv]);
@@ -483,7 +488,10 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   } else {
     regs_claim<kRegsSoftmax>();
     // ======================= softmax + epilogue =======================
-    const int grp = (warp - 4) >> 2;                // 0: even tiles, 1: odd tiles
+    // Both groups work on every key tile: group g takes its keys
+    // [64g, 64g + 64) with a running max / sum of its own and accumulates
+    // into O_g; the two partial softmaxes are merged per row at the end.
+    const int grp = (warp - 4) >> 2;
     const int wq = warp & 3;
     const int m = wq * 32 + lane;                   // packed row = TMEM lane
     const int r = r0 + m / p.g;
@@ -491,32 +499,32 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     const bool row_ok = r <= r_hi;
     const int limit = !row_ok ? kv_end : (mode == ZARYA_MASK_SLOT_CAUSAL ? P + r + 1 : P + R);
     const uint32_t t_row = tmem + (static_cast<uint32_t>(wq * 32) << 16);
-    const uint32_t t_s = t_row + grp * 128;
     const uint32_t t_o = t_row + kTmemO + grp * 128;
     const float sl2 = p.scale_log2;
     float m_run = -INFINITY;  // running max, in scaled log2 units
     float l_run = 0.f;
     bool ok = true;
 
-    for (int i = grp; i < nt; i += 2) {
-      const int j = i >> 1;
-      const int c0 = (t_begin + i) * kBlockN;
-      if (ok) ok = wait_bar(&bars->s_full[grp], j & 1, bars, p.err);
+    for (int i = 0; i < nt; ++i) {
+      const int sb = i & 1;
+      const int c0 = (t_begin + i) * kBlockN + grp * 64;   // first key of this half
+      const uint32_t t_s = t_row + sb * 128 + grp * 64;
+      if (ok) ok = wait_bar(&bars->s_full[sb], (i >> 1) & 1, bars, p.err);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
-      float s[128];
-      tmem_ld_32x32b_x128(t_s, s);
+      float s[64];
+      tmem_ld_32x32b_x64(t_s, s);
 
-      if (c0 + kBlockN > limit) {
+      if (c0 + 64 > limit) {
 #pragma unroll
-        for (int x = 0; x < 128; ++x)
+        for (int x = 0; x < 64; ++x)
           if (c0 + x >= limit) s[x] = -INFINITY;
       }
       float mx[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) mx[k] = s[k];
 #pragma unroll
-      for (int x = 8; x < 128; x += 8)
+      for (int x = 8; x < 64; x += 8)
 #pragma unroll
         for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], s[x + k]);
       const float mt4 = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
@@ -532,9 +540,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       }
       const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
 
-      // O may be rescaled here: S(i) being complete means this group's
-      // previous P*V (issued before Q*K^T(i)) is complete as well.
-      if (warp_need && j > 0) {
+      // Rescaling O_g must wait for P*V(i-1), the last MMA that wrote it.
+      // S(i) complete implies P*V(i-2) complete (issued before Q*K^T(i)), so
+      // this parity wait on o_done[(i-1) & 1] cannot alias an older phase.
+      if (warp_need && i > 0) {
+        if (ok) ok = wait_bar(&bars->o_done[(i - 1) & 1], ((i - 1) >> 1) & 1, bars, p.err);
+        tc_fence_after();
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
           float v[32];
@@ -547,12 +558,14 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       }
       // Keys at or past kv_end in the last tile: their V rows (stale smem,
       // unloaded pages or another sequence's cache) must be exact zeros, or a
-      // NaN there would poison P*V even with P = 0.
-      if (c0 + kBlockN > kv_end) {
+      // NaN there would poison P*V even with P = 0. Each group clears the
+      // rows of its own half.
+      if (c0 + 64 > kv_end) {
         const int sv = i % kStagesV;
         if (ok) ok = wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err);
-        if (ok && c0 + m >= kv_end) {
-          uint8_t* vrow = smem + kOffV + sv * kTileBytes + (m >> 3) * 1024 + (m & 7) * 128;
+        const int key = grp * 64 + (m & 63);
+        if (ok && m < 64 && c0 + (m & 63) >= kv_end) {
+          uint8_t* vrow = smem + kOffV + sv * kTileBytes + (key >> 3) * 1024 + (key & 7) * 128;
           const uint4 z = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
           for (int x = 0; x < 8; ++x) {
@@ -563,43 +576,35 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         // the zeros are generic-proxy writes; P*V reads V through the async proxy
         fence_proxy_async_smem();
       }
-      // P = 2^(s * scale * log2 e - m) as packed bf16 pairs over the first 64
-      // columns of this group's S buffer (S is already in registers).
+      // P = 2^(s * scale * log2 e - m) as packed bf16 pairs over the first 32
+      // columns of this group's half of the S buffer (S is in registers).
+      float pk[32];
       float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
 #pragma unroll
-      for (int ch = 0; ch < 2; ++ch) {
-        float pk[32];
-#pragma unroll
-        for (int x = 0; x < 32; x += 2) {
-          const int c = ch * 64 + 2 * x;
-          const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
-          const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
-          const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
-          const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
-          rs0 += e0;
-          rs1 += e1;
-          rs2 += e2;
-          rs3 += e3;
-          pk[x] = __uint_as_float(pack_bf16(e0, e1));
-          pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
-        }
-        tmem_st_32x32b_x32(t_s + ch * 32, pk);
+      for (int x = 0; x < 32; x += 2) {
+        const int c = 2 * x;
+        const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
+        const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
+        const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
+        const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
+        rs0 += e0;
+        rs1 += e1;
+        rs2 += e2;
+        rs3 += e3;
+        pk[x] = __uint_as_float(pack_bf16(e0, e1));
+        pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
       }
+      tmem_st_32x32b_x32(t_s, pk);
       l_run += (rs0 + rs1) + (rs2 + rs3);
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->p_full[grp]);
+      if (lane == 0) mbar_arrive(&bars->p_full[sb]);
     }
 
     // ---- epilogue: merge the two groups' partial results per row ----
-    const int n0 = (nt + 1) >> 1;   // tiles of group 0
-    const int n1 = nt >> 1;         // tiles of group 1
-    const int n_mine = grp == 0 ? n0 : n1;
-    // Each group waits for its own last P*V (its previous one completed before
-    // its last S, so this parity wait cannot alias an older phase); a group may
-    // own no tile when nt == 1. The barrier below then joins both groups: the
-    // last MMA of the CTA is one of the two, so every MMA has completed.
-    if (n_mine > 0 && ok) ok = wait_bar(&bars->o_done[grp], (n_mine - 1) & 1, bars, p.err);
+    // The last P*V completes after every other MMA of the CTA; P*V(nt-3) is
+    // known complete, so the parity wait cannot alias an older phase.
+    if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p.err);
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_before();
     named_bar_sync(1, 256);
@@ -631,15 +636,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
 #pragma unroll
     for (int ch = 0; ch < 2; ++ch) {
       float va[32], vb[32];
-      if (ok && n0 > 0) tmem_ld_32x32b_x32(t_row + kTmemO + col0 + ch * 32, va);
-      else {
+      if (ok) {
+        tmem_ld_32x32b_x32(t_row + kTmemO + col0 + ch * 32, va);
+        tmem_ld_32x32b_x32(t_row + kTmemO + 128 + col0 + ch * 32, vb);
+      } else {
 #pragma unroll
-        for (int x = 0; x < 32; ++x) va[x] = 0.f;
-      }
-      if (ok && n1 > 0) tmem_ld_32x32b_x32(t_row + kTmemO + 128 + col0 + ch * 32, vb);
-      else {
-#pragma unroll
-        for (int x = 0; x < 32; ++x) vb[x] = 0.f;
+        for (int x = 0; x < 32; ++x) va[x] = vb[x] = 0.f;
       }
 #pragma unroll
       for (int x = 0; x < 32; ++x) o[ch * 32 + x] = wA * va[x] + wB * vb[x];
