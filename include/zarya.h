@@ -180,6 +180,23 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
                              const zarya_attn_desc* desc, zarya_stream_t stream);
 
 /*
+ * The ZARYA_APPEND_COMMIT form of zarya_kv_append with the advanced lengths
+ * going to a second array: the same rows are copied to positions
+ * cache_lens[b] + i, and new_lens[b] (device [B]) receives
+ * cache_lens[b] + accept_len[b] for every sequence that passed the device
+ * checks (others keep their new_lens entry and set the error word).
+ * cache_lens is only read. new_lens may be cache_lens itself, which is then
+ * exactly zarya_kv_append(..., ZARYA_APPEND_COMMIT, ...). A caller that keeps
+ * the lengths of consecutive steps in two arrays (ping-pong) needs no copy
+ * between steps. Not a step of the paper's method, only a form of step 7.
+ */
+zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
+                                       const int32_t* accept_len, void* k_cache, void* v_cache,
+                                       const int32_t* cache_lens, int32_t* new_lens,
+                                       const int32_t* page_table, const zarya_attn_desc* desc,
+                                       zarya_stream_t stream);
+
+/*
  * Synchronises `stream`, then reads and clears the error word of the device
  * that owns it. Returns ZARYA_OK when it was clear, ZARYA_ERR_DEVICE_FAULT
  * when it was set (*code receives its ZARYA_DEVERR_* value; code may be

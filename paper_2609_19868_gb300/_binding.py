@@ -75,6 +75,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_slot_attn_noalloc.restype = ctypes.c_int
     lib.zarya_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, dp, vp]
     lib.zarya_kv_append.restype = ctypes.c_int
+    lib.zarya_kv_append_commit_to.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, dp, vp]
+    lib.zarya_kv_append_commit_to.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
     lib.zarya_check_device_error.restype = ctypes.c_int
     lib.zarya_last_error.argtypes = []
@@ -205,6 +207,26 @@ def kv_append(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, page_table
                                 _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_kv_append")
+
+
+def kv_append_commit_to(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, new_lens,
+                        page_table, desc: AttnDesc, stream=None) -> None:
+    """``zarya_kv_append_commit_to``: the commit with new_lens = cache_lens + accept_len
+    written to a second array (cache_lens is only read)."""
+    for name, t in (("k_new", k_new), ("v_new", v_new), ("k_cache", k_cache),
+                    ("v_cache", v_cache)):
+        _check_cuda(name, t)
+    _check_cuda("accept_len", accept_len, torch.int32)
+    _check_cuda("cache_lens", cache_lens, torch.int32)
+    _check_cuda("new_lens", new_lens, torch.int32)
+    if page_table is not None:
+        _check_cuda("page_table", page_table, torch.int32)
+    st = load().zarya_kv_append_commit_to(_ptr(k_new), _ptr(v_new), _ptr(accept_len),
+                                          _ptr(k_cache), _ptr(v_cache), _ptr(cache_lens),
+                                          _ptr(new_lens), _ptr(page_table), ctypes.byref(desc),
+                                          _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_kv_append_commit_to")
 
 
 def check_device_error(stream=None) -> int:

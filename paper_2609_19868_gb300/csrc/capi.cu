@@ -333,15 +333,17 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching slot_attn_tc_kernel", ce);
 }
 
-zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
-                             void* k_cache, void* v_cache, int32_t* cache_lens,
-                             const int32_t* page_table, int32_t flags,
-                             const zarya_attn_desc* desc, zarya_stream_t stream_) {
+namespace {
+
+zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t* accept_len,
+                            void* k_cache, void* v_cache, const int32_t* cache_lens,
+                            int32_t* new_lens, const int32_t* page_table, bool commit,
+                            const zarya_attn_desc* desc, zarya_stream_t stream_) {
   zarya_status st = check_desc(desc);
   if (st != ZARYA_OK) return st;
-  if (flags != ZARYA_APPEND_STAGE && flags != ZARYA_APPEND_COMMIT) return ZARYA_ERR_INVALID_ARG;
   if (!k_new || !v_new || !accept_len || !k_cache || !v_cache || !cache_lens)
     return ZARYA_ERR_INVALID_ARG;
+  if (commit && !new_lens) return ZARYA_ERR_INVALID_ARG;
   if ((desc->page_size > 0) != (page_table != nullptr)) return ZARYA_ERR_INVALID_ARG;
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
     return ZARYA_ERR_INVALID_ARG;
@@ -358,6 +360,7 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
   p.k_cache = k_cache;
   p.v_cache = v_cache;
   p.cache_lens = cache_lens;
+  p.new_lens = new_lens;
   p.page_table = page_table;
   p.q_row_offsets = desc->q_row_offsets;
   p.err = err;
@@ -370,8 +373,29 @@ zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t
   p.max_pages = desc->page_size > 0 ? desc->cache_capacity / desc->page_size : 0;
   p.n_pages = desc->n_pages;
   if (desc->batch > 65535) return ZARYA_ERR_UNSUPPORTED;
-  ce = launch_kv_append(p, flags == ZARYA_APPEND_COMMIT, stream);
-  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the append kernels", ce);
+  ce = launch_kv_append(p, commit, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the append kernel", ce);
+}
+
+}  // namespace
+
+zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
+                             void* k_cache, void* v_cache, int32_t* cache_lens,
+                             const int32_t* page_table, int32_t flags,
+                             const zarya_attn_desc* desc, zarya_stream_t stream) {
+  if (flags != ZARYA_APPEND_STAGE && flags != ZARYA_APPEND_COMMIT) return ZARYA_ERR_INVALID_ARG;
+  const bool commit = flags == ZARYA_APPEND_COMMIT;
+  return kv_append_impl(k_new, v_new, accept_len, k_cache, v_cache, cache_lens,
+                        commit ? cache_lens : nullptr, page_table, commit, desc, stream);
+}
+
+zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
+                                       const int32_t* accept_len, void* k_cache, void* v_cache,
+                                       const int32_t* cache_lens, int32_t* new_lens,
+                                       const int32_t* page_table, const zarya_attn_desc* desc,
+                                       zarya_stream_t stream) {
+  return kv_append_impl(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, new_lens,
+                        page_table, true, desc, stream);
 }
 
 zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {

@@ -65,13 +65,15 @@ struct AppendParams {
   const int32_t* accept_len;
   void* k_cache;
   void* v_cache;
-  int32_t* cache_lens;
+  const int32_t* cache_lens;
+  int32_t* new_lens;        // commit: receives cache_lens[b] + accept_len[b] (may alias cache_lens)
   const int32_t* page_table;
   const int32_t* q_row_offsets;
   int* err;
   int B, row_bytes;  // row_bytes = Hkv * D * element size (multiple of 16)
   int max_rows, total_rows, capacity;
   int page_size, max_pages, n_pages;
+  int rows_per_block;       // block rows copied by one CTA (gridDim.x CTAs per sequence)
 };
 
 // Dynamic shared memory of the tensor-core kernel.
@@ -91,8 +93,10 @@ size_t workspace_counter_bytes(const zarya_attn_desc* desc);
 // kernel's set-up can overlap the tail of the kernel before it.
 struct PdlLaunch {
   cudaLaunchConfig_t cfg;
-  cudaLaunchAttribute attr[1];
-  PdlLaunch(dim3 grid, dim3 block, size_t smem, cudaStream_t stream) : cfg{}, attr{} {
+  cudaLaunchAttribute attr[2];
+  // cluster_x > 1: thread-block clusters of cluster_x CTAs along x.
+  PdlLaunch(dim3 grid, dim3 block, size_t smem, cudaStream_t stream, unsigned cluster_x = 1)
+      : cfg{}, attr{} {
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
@@ -101,6 +105,13 @@ struct PdlLaunch {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (cluster_x > 1) {
+      attr[1].id = cudaLaunchAttributeClusterDimension;
+      attr[1].val.clusterDim.x = cluster_x;
+      attr[1].val.clusterDim.y = 1;
+      attr[1].val.clusterDim.z = 1;
+      cfg.numAttrs = 2;
+    }
   }
 };
 

@@ -131,11 +131,18 @@ slot_attn_f32_kernel(const SimtParams p) {
   for (int x = 0; x < kPerLane; ++x) out[lane + 32 * x] = o[x] / l;
 }
 
-constexpr int kAppendRowsPerBlock = 8;
+// At most this many CTAs share one sequence's rows, so that a commit can
+// advance cache_lens[b] inside one thread-block cluster.
+constexpr int kAppendMaxCtasPerSeq = 8;
+constexpr int kAppendThreads = 256;
+constexpr int kAppendUnroll = 4;   // 16-byte vectors of K and of V in flight per thread
 
-// Copies rows i < accept_len[b] of the block (chunk blockIdx.x of
-// kAppendRowsPerBlock rows, sequence blockIdx.y) to cache positions P_b + i.
-__global__ void __launch_bounds__(256)
+// Copies rows i < accept_len[b] of the block (rows [x * rows_per_block, ...)
+// for CTA x, sequence blockIdx.y) to cache positions P_b + i. With `commit`
+// the CTAs of a sequence form one cluster: after every CTA has read P_b and
+// copied its rows, CTA 0 writes new_lens[b] = P_b + accept_len[b].
+template <bool kCommit>
+__global__ void __launch_bounds__(kAppendThreads)
 kv_append_copy_kernel(const AppendParams p) {
   grid_dependency_wait();
   grid_launch_dependents();
@@ -150,53 +157,59 @@ kv_append_copy_kernel(const AppendParams p) {
   else if (P < 0 || static_cast<long long>(P) + a > p.capacity) code = ZARYA_DEVERR_CAPACITY;
   if (code != 0) {
     if (blockIdx.x == 0 && threadIdx.x == 0) record_error(p.err, code);
-    return;
-  }
-  const int i0 = blockIdx.x * kAppendRowsPerBlock;
-  if (i0 >= a) return;
-  const int n_rows = min(kAppendRowsPerBlock, a - i0);
-  const int vec_per_row = p.row_bytes >> 4;
-  const uint4* kn = reinterpret_cast<const uint4*>(p.k_new);
-  const uint4* vn = reinterpret_cast<const uint4*>(p.v_new);
-  uint4* kc = reinterpret_cast<uint4*>(p.k_cache);
-  uint4* vc = reinterpret_cast<uint4*>(p.v_cache);
-  const int total = n_rows * vec_per_row;
-  for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
-    const int ri = idx / vec_per_row;
-    const int v = idx - ri * vec_per_row;
-    const int i = i0 + ri;
-    const int t = P + i;
-    long long tr;
-    if (p.page_size == 0) {
-      tr = static_cast<long long>(b) * p.capacity + t;
-    } else {
-      const int page = p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
-      if (page < 0 || page >= p.n_pages) {
-        record_error(p.err, ZARYA_DEVERR_PAGE_ID);
-        continue;
+  } else {
+    const int i0 = blockIdx.x * p.rows_per_block;
+    const int n_rows = max(0, min(p.rows_per_block, a - i0));
+    const int vec_per_row = p.row_bytes >> 4;
+    const uint4* kn = reinterpret_cast<const uint4*>(p.k_new);
+    const uint4* vn = reinterpret_cast<const uint4*>(p.v_new);
+    uint4* kc = reinterpret_cast<uint4*>(p.k_cache);
+    uint4* vc = reinterpret_cast<uint4*>(p.v_cache);
+    const int total = n_rows * vec_per_row;
+    for (int base = 0; base < total; base += kAppendUnroll * kAppendThreads) {
+      uint4 kv[kAppendUnroll], vv[kAppendUnroll];
+      long long dst[kAppendUnroll];
+      // all loads first, then all stores: kAppendUnroll round trips overlap
+#pragma unroll
+      for (int u = 0; u < kAppendUnroll; ++u) {
+        const int idx = base + u * kAppendThreads + threadIdx.x;
+        dst[u] = -1;
+        if (idx < total) {
+          const int ri = idx / vec_per_row;
+          const int v = idx - ri * vec_per_row;
+          const int i = i0 + ri;
+          const int t = P + i;
+          long long tr = -1;
+          if (p.page_size == 0) {
+            tr = static_cast<long long>(b) * p.capacity + t;
+          } else {
+            const int page = p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
+            if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+            else tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+          }
+          if (tr >= 0) {
+            const long long src = static_cast<long long>(row0 + i) * vec_per_row + v;
+            kv[u] = __ldg(kn + src);
+            vv[u] = __ldg(vn + src);
+            dst[u] = tr * vec_per_row + v;
+          }
+        }
       }
-      tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+#pragma unroll
+      for (int u = 0; u < kAppendUnroll; ++u) {
+        if (dst[u] >= 0) {
+          kc[dst[u]] = kv[u];
+          vc[dst[u]] = vv[u];
+        }
+      }
     }
-    const long long src = static_cast<long long>(row0 + i) * vec_per_row + v;
-    const long long dst = tr * vec_per_row + v;
-    kc[dst] = __ldg(kn + src);
-    vc[dst] = __ldg(vn + src);
   }
-}
-
-// cache_lens[b] += accept_len[b] for every sequence whose copy was valid.
-__global__ void kv_append_advance_kernel(const AppendParams p) {
-  grid_dependency_wait();
-  grid_launch_dependents();
-  for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < p.B; b += gridDim.x * blockDim.x) {
-    const int a = p.accept_len[b];
-    const int P = p.cache_lens[b];
-    const int row0 = p.q_row_offsets[b];
-    const int R = p.q_row_offsets[b + 1] - row0;
-    if (R < 0 || R > p.max_rows || row0 < 0 || row0 + R > p.total_rows || a < 0 || a > R || P < 0 ||
-        static_cast<long long>(P) + a > p.capacity)
-      continue;
-    p.cache_lens[b] = P + a;
+  if (kCommit) {
+    // Every CTA of this sequence has read cache_lens[b] before it changes
+    // (new_lens may alias cache_lens).
+    cluster_arrive();
+    cluster_wait();
+    if (code == 0 && blockIdx.x == 0 && threadIdx.x == 0) p.new_lens[b] = P + a;
   }
 }
 
@@ -222,19 +235,17 @@ cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream) {
   }
 }
 
-cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream) {
-  const int chunks = (p.max_rows + kAppendRowsPerBlock - 1) / kAppendRowsPerBlock;
-  if (chunks > 0) {
-    PdlLaunch l(dim3(chunks, p.B), dim3(256), 0, stream);
-    cudaError_t e = cudaLaunchKernelEx(&l.cfg, kv_append_copy_kernel, p);
-    if (e != cudaSuccess) return e;
-  }
+cudaError_t launch_kv_append(const AppendParams& p_in, bool commit, cudaStream_t stream) {
+  AppendParams p = p_in;
+  const int rows = p.max_rows > 0 ? p.max_rows : 1;
+  p.rows_per_block = max(8, (rows + kAppendMaxCtasPerSeq - 1) / kAppendMaxCtasPerSeq);
+  const int ctas = (rows + p.rows_per_block - 1) / p.rows_per_block;   // <= 8
   if (commit) {
-    const int block = 128;
-    PdlLaunch l(dim3((p.B + block - 1) / block), dim3(block), 0, stream);
-    return cudaLaunchKernelEx(&l.cfg, kv_append_advance_kernel, p);
+    PdlLaunch l(dim3(ctas, p.B), dim3(kAppendThreads), 0, stream, static_cast<unsigned>(ctas));
+    return cudaLaunchKernelEx(&l.cfg, kv_append_copy_kernel<true>, p);
   }
-  return cudaSuccess;
+  PdlLaunch l(dim3(ctas, p.B), dim3(kAppendThreads), 0, stream);
+  return cudaLaunchKernelEx(&l.cfg, kv_append_copy_kernel<false>, p);
 }
 
 }  // namespace zarya

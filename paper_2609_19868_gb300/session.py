@@ -50,9 +50,16 @@ class DeviceBatch:
                      self.n_slots, self.slot_len, self.mask_mode, self.out, self.desc,
                      self.workspace, stream=stream)
 
-    def commit(self, stream=None) -> None:
-        zb.kv_append(self.k_new, self.v_new, self.accept_len, self.k_cache, self.v_cache,
-                     self.cache_lens, self.page_table, self.desc, commit=True, stream=stream)
+    def commit(self, stream=None, new_lens=None) -> None:
+        """Append the accepted rows and advance the lengths: in place, or into
+        ``new_lens`` (leaving ``cache_lens`` as it was) when given."""
+        if new_lens is None:
+            zb.kv_append(self.k_new, self.v_new, self.accept_len, self.k_cache, self.v_cache,
+                         self.cache_lens, self.page_table, self.desc, commit=True, stream=stream)
+        else:
+            zb.kv_append_commit_to(self.k_new, self.v_new, self.accept_len, self.k_cache,
+                                   self.v_cache, self.cache_lens, new_lens, self.page_table,
+                                   self.desc, stream=stream)
 
 
 def _i32(a, device) -> torch.Tensor:

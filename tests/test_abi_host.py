@@ -139,3 +139,18 @@ def test_append_rejects_invalid_calls(lib):
     assert app(k_new=FAKE + 4) == 1
     assert app(page_table=FAKE) == 1
     assert app(desc=_desc(n_kv_heads=1, n_q_heads=1, head_dim=4)) == 2  # row not 16-byte multiple
+
+
+def test_commit_to_rejects_invalid_calls(lib):
+    vp = ctypes.c_void_p
+    d = _desc()
+
+    def app(new_lens=FAKE, cache_lens=FAKE, desc=d, k_cache=FAKE):
+        return lib.zarya_kv_append_commit_to(vp(FAKE), vp(FAKE), vp(FAKE), vp(k_cache), vp(FAKE),
+                                             vp(cache_lens), vp(new_lens), vp(None),
+                                             None if desc is None else ctypes.byref(desc), None)
+
+    assert app(new_lens=None) == 1
+    assert app(cache_lens=None) == 1
+    assert app(desc=None) == 1
+    assert app(k_cache=FAKE + 8) == 1

@@ -65,6 +65,42 @@ def test_stage_then_commit_bit_exact(zs, oracle_mod, name, small):
     assert np.array_equal(db.cache_lens.cpu().numpy(), lens2)
 
 
+@pytest.mark.parametrize("name,small", [("decode_small", True), ("serving_mix", True),
+                                        ("serving_mix", False)])
+def test_commit_to_second_array_leaves_lengths_alone(zs, oracle_mod, name, small):
+    """zarya_kv_append_commit_to: the same rows as an in-place commit, the
+    advanced lengths in new_lens, cache_lens untouched."""
+    session, zb = zs
+    w = wl.make(name, small=small)
+    db = session.upload(w, "cuda")
+    db.stage()
+    new_lens = torch.full_like(db.cache_lens, -7)
+    db.commit(new_lens=new_lens)
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    _, _, kc2, vc2, lens2 = _oracle_stage_commit(oracle_mod, w)
+    gk, gv = _bits(db.k_cache), _bits(db.v_cache)
+    assert np.array_equal(gk, kc2.view(gk.dtype))
+    assert np.array_equal(gv, vc2.view(gv.dtype))
+    assert np.array_equal(db.cache_lens.cpu().numpy(), w.cache_lens)
+    assert np.array_equal(new_lens.cpu().numpy(), lens2)
+
+
+def test_commit_to_skips_a_failing_sequence(zs):
+    session, zb = zs
+    w = wl.make("decode_small", small=True)
+    db = session.upload(w, "cuda")
+    db.accept_len[1] = int(w.R[1]) + 1
+    new_lens = torch.full_like(db.cache_lens, -7)
+    db.commit(new_lens=new_lens)
+    assert zb.check_device_error() == 4
+    got = new_lens.cpu().numpy()
+    assert got[1] == -7
+    for b in range(w.B):
+        if b != 1:
+            assert got[b] == w.cache_lens[b] + w.accept_len[b]
+
+
 def test_commit_of_nothing_is_a_noop(zs):
     session, zb = zs
     w = wl.make("decode_small", small=True)
