@@ -134,6 +134,26 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
                              zarya_stream_t stream);
 
 /*
+ * The block's own K/V staged and attended in one launch: exactly
+ * zarya_kv_append(k_new, v_new, <R_b for every b>, ..., ZARYA_APPEND_STAGE)
+ * followed by zarya_slot_attn(...) on the same stream (Sec. 5.2 step 3: the
+ * block attends over the cached prefix plus itself, its K/V coming from the
+ * same forward pass). k_new / v_new are [total_rows, Hkv, D] like the append's;
+ * block row i of sequence b is written to cache position P_b + i (through the
+ * page table when paged) and cache_lens is left alone. On the tensor-core path
+ * the CTAs that read a block row copy it into the cache themselves just before
+ * loading it, so the copy overlaps the streaming of the prefix. Arguments,
+ * workspace and errors as zarya_slot_attn; k_new / v_new must be non-NULL and
+ * 16-byte aligned.
+ */
+zarya_status zarya_slot_attn_staged(const void* q, const void* k_new, const void* v_new,
+                                    void* k_cache, void* v_cache, const int32_t* cache_lens,
+                                    const int32_t* page_table, const int32_t* n_slots,
+                                    const int32_t* slot_len, const int32_t* mask_mode, void* out,
+                                    void* workspace, size_t workspace_bytes,
+                                    const zarya_attn_desc* desc, zarya_stream_t stream);
+
+/*
  * zarya_slot_attn without a workspace argument, for callers that cannot
  * allocate device memory at the point where they run attention: a serving
  * engine that has already given all of HBM to its own cache pool, a host

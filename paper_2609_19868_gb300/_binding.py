@@ -71,6 +71,9 @@ def load() -> ctypes.CDLL:
     lib.zarya_slot_attn_workspace_size.restype = sz
     lib.zarya_slot_attn.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, dp, vp]
     lib.zarya_slot_attn.restype = ctypes.c_int
+    lib.zarya_slot_attn_staged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
+                                           dp, vp]
+    lib.zarya_slot_attn_staged.restype = ctypes.c_int
     lib.zarya_slot_attn_noalloc.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, dp, vp]
     lib.zarya_slot_attn_noalloc.restype = ctypes.c_int
     lib.zarya_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, dp, vp]
@@ -167,6 +170,32 @@ def slot_attn(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len, ma
                                 ctypes.byref(desc), _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_slot_attn")
+
+
+def slot_attn_staged(q, k_new, v_new, k_cache, v_cache, cache_lens, page_table, n_slots,
+                     slot_len, mask_mode, out, desc: AttnDesc,
+                     workspace: Optional[torch.Tensor] = None, stream=None) -> None:
+    """``zarya_slot_attn_staged``: stage the block's own K/V into the cache
+    and attend, in one launch (= stage append + ``zarya_slot_attn``)."""
+    for name, t in (("q", q), ("k_new", k_new), ("v_new", v_new), ("k_cache", k_cache),
+                    ("v_cache", v_cache), ("out", out)):
+        _check_cuda(name, t)
+    for name, t in (("cache_lens", cache_lens), ("n_slots", n_slots), ("slot_len", slot_len),
+                    ("mask_mode", mask_mode)):
+        _check_cuda(name, t, torch.int32)
+    if page_table is not None:
+        _check_cuda("page_table", page_table, torch.int32)
+    ws_bytes = 0
+    if workspace is not None:
+        _check_cuda("workspace", workspace)
+        ws_bytes = workspace.numel() * workspace.element_size()
+    st = load().zarya_slot_attn_staged(_ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache),
+                                       _ptr(v_cache), _ptr(cache_lens), _ptr(page_table),
+                                       _ptr(n_slots), _ptr(slot_len), _ptr(mask_mode), _ptr(out),
+                                       _ptr(workspace), ws_bytes, ctypes.byref(desc),
+                                       _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_slot_attn_staged")
 
 
 def slot_attn_noalloc(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len,

@@ -200,21 +200,39 @@ size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc) {
   return plan_tc(desc, sm_count()).bytes;
 }
 
-zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_cache,
-                             const int32_t* cache_lens, const int32_t* page_table,
-                             const int32_t* n_slots, const int32_t* slot_len,
-                             const int32_t* mask_mode, void* out, void* workspace,
-                             size_t workspace_bytes, const zarya_attn_desc* desc,
-                             zarya_stream_t stream_) {
+namespace {
+
+zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t* accept_len,
+                            void* k_cache, void* v_cache, const int32_t* cache_lens,
+                            int32_t* new_lens, const int32_t* page_table, bool commit,
+                            const zarya_attn_desc* desc, zarya_stream_t stream_);
+
+// Attention, optionally staging the block's own K/V (k_new / v_new) first.
+zarya_status slot_attn_impl(const void* q, const void* k_new, const void* v_new,
+                            const void* k_cache, const void* v_cache, const int32_t* cache_lens,
+                            const int32_t* page_table, const int32_t* n_slots,
+                            const int32_t* slot_len, const int32_t* mask_mode, void* out,
+                            void* workspace, size_t workspace_bytes, const zarya_attn_desc* desc,
+                            zarya_stream_t stream_) {
   zarya_status st = check_desc(desc);
   if (st != ZARYA_OK) return st;
   st = check_attn_support(desc);
   if (st != ZARYA_OK) return st;
   if (!q || !k_cache || !v_cache || !cache_lens || !n_slots || !slot_len || !mask_mode || !out)
     return ZARYA_ERR_INVALID_ARG;
+  const bool staged = k_new != nullptr || v_new != nullptr;
+  if (staged && (!k_new || !v_new || !aligned16(k_new) || !aligned16(v_new)))
+    return ZARYA_ERR_INVALID_ARG;
   if ((desc->page_size > 0) != (page_table != nullptr)) return ZARYA_ERR_INVALID_ARG;
   if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
     return ZARYA_ERR_INVALID_ARG;
+  if (staged && desc->dtype == ZARYA_FP32) {
+    // The CUDA-core path stages with the append kernel, then attends.
+    st = kv_append_impl(k_new, v_new, nullptr, const_cast<void*>(k_cache),
+                        const_cast<void*>(v_cache), cache_lens, nullptr, page_table, false, desc,
+                        stream_);
+    if (st != ZARYA_OK) return st;
+  }
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   cudaError_t ce = select_device(stream, q);
   if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
@@ -329,11 +347,13 @@ zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_c
   p.splits = plan.splits;
   p.cluster = (plan.splits > 1 && plan.splits <= kMaxClusterSplits) ? 1 : 0;
   p.scale_log2 = scale * 1.4426950408889634f;
+  p.k_new = k_new;
+  p.v_new = v_new;
+  p.k_cache = const_cast<void*>(k_cache);
+  p.v_cache = const_cast<void*>(v_cache);
   ce = launch_slot_attn_tc(map_q, map_k, map_v, p, stream);
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching slot_attn_tc_kernel", ce);
 }
-
-namespace {
 
 zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t* accept_len,
                             void* k_cache, void* v_cache, const int32_t* cache_lens,
@@ -341,8 +361,8 @@ zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t*
                             const zarya_attn_desc* desc, zarya_stream_t stream_) {
   zarya_status st = check_desc(desc);
   if (st != ZARYA_OK) return st;
-  if (!k_new || !v_new || !accept_len || !k_cache || !v_cache || !cache_lens)
-    return ZARYA_ERR_INVALID_ARG;
+  // accept_len == nullptr (internal use only): copy every block row
+  if (!k_new || !v_new || !k_cache || !v_cache || !cache_lens) return ZARYA_ERR_INVALID_ARG;
   if (commit && !new_lens) return ZARYA_ERR_INVALID_ARG;
   if ((desc->page_size > 0) != (page_table != nullptr)) return ZARYA_ERR_INVALID_ARG;
   if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
@@ -379,11 +399,33 @@ zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t*
 
 }  // namespace
 
+zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_cache,
+                             const int32_t* cache_lens, const int32_t* page_table,
+                             const int32_t* n_slots, const int32_t* slot_len,
+                             const int32_t* mask_mode, void* out, void* workspace,
+                             size_t workspace_bytes, const zarya_attn_desc* desc,
+                             zarya_stream_t stream) {
+  return slot_attn_impl(q, nullptr, nullptr, k_cache, v_cache, cache_lens, page_table, n_slots,
+                        slot_len, mask_mode, out, workspace, workspace_bytes, desc, stream);
+}
+
+zarya_status zarya_slot_attn_staged(const void* q, const void* k_new, const void* v_new,
+                                    void* k_cache, void* v_cache, const int32_t* cache_lens,
+                                    const int32_t* page_table, const int32_t* n_slots,
+                                    const int32_t* slot_len, const int32_t* mask_mode, void* out,
+                                    void* workspace, size_t workspace_bytes,
+                                    const zarya_attn_desc* desc, zarya_stream_t stream) {
+  if (!k_new || !v_new) return ZARYA_ERR_INVALID_ARG;
+  return slot_attn_impl(q, k_new, v_new, k_cache, v_cache, cache_lens, page_table, n_slots,
+                        slot_len, mask_mode, out, workspace, workspace_bytes, desc, stream);
+}
+
 zarya_status zarya_kv_append(const void* k_new, const void* v_new, const int32_t* accept_len,
                              void* k_cache, void* v_cache, int32_t* cache_lens,
                              const int32_t* page_table, int32_t flags,
                              const zarya_attn_desc* desc, zarya_stream_t stream) {
   if (flags != ZARYA_APPEND_STAGE && flags != ZARYA_APPEND_COMMIT) return ZARYA_ERR_INVALID_ARG;
+  if (!accept_len) return ZARYA_ERR_INVALID_ARG;
   const bool commit = flags == ZARYA_APPEND_COMMIT;
   return kv_append_impl(k_new, v_new, accept_len, k_cache, v_cache, cache_lens,
                         commit ? cache_lens : nullptr, page_table, commit, desc, stream);
@@ -394,6 +436,7 @@ zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
                                        const int32_t* cache_lens, int32_t* new_lens,
                                        const int32_t* page_table, const zarya_attn_desc* desc,
                                        zarya_stream_t stream) {
+  if (!accept_len) return ZARYA_ERR_INVALID_ARG;
   return kv_append_impl(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, new_lens,
                         page_table, true, desc, stream);
 }

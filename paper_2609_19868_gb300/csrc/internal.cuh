@@ -38,6 +38,13 @@ struct TcParams {
   int m_tiles, splits;
   int cluster;        // 1: the splits of a tile form a cluster and merge through DSMEM
   float scale_log2;   // softmax scale * log2(e)
+  // Staged attention: when k_new != nullptr, block row i of sequence b
+  // (k_new / v_new row q_row_offsets[b] + i) is first written to cache
+  // position P_b + i by the CTAs that read it.
+  const void* k_new;  // bf16 [total_rows, Hkv, D] or nullptr
+  const void* v_new;
+  void* k_cache;      // bf16 cache (the tensor maps' base addresses)
+  void* v_cache;
 };
 
 // Parameters of the fp32 CUDA-core path and of the append kernels.

@@ -147,10 +147,10 @@ kv_append_copy_kernel(const AppendParams p) {
   grid_dependency_wait();
   grid_launch_dependents();
   const int b = blockIdx.y;
-  const int a = p.accept_len[b];
   const int P = p.cache_lens[b];
   const int row0 = p.q_row_offsets[b];
   const int R = p.q_row_offsets[b + 1] - row0;
+  const int a = p.accept_len != nullptr ? p.accept_len[b] : R;   // nullptr: the whole block
   int code = 0;
   if (R < 0 || R > p.max_rows || row0 < 0 || row0 + R > p.total_rows) code = ZARYA_DEVERR_ROWS;
   else if (a < 0 || a > R) code = ZARYA_DEVERR_ACCEPT;

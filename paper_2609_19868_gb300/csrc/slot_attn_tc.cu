@@ -80,6 +80,7 @@ struct Bars {
   uint64_t o_done[2];   // o_done[i & 1], phase i >> 1: P*V(i) has completed
   uint64_t drain;
   uint64_t kfree;   // this CTA's last Q*K^T has completed: its K ring is idle
+  uint64_t staged;  // staged attention: the block rows this CTA reads are in the cache
   uint64_t ready;   // cluster merge: every partial row this CTA owns has landed
   uint64_t go;      // cluster merge: every other split's K ring is free to receive
   uint32_t tmem_base;
@@ -226,11 +227,68 @@ __device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity,
   return false;
 }
 
+// Staged attention: copy block rows [i_lo, i_hi) of sequence b, KV head kvh,
+// of K and V from k_new / v_new ([total_rows, Hkv, D]) to cache positions
+// P + i (the 256 softmax threads, idle until the first S tile; 16-byte
+// vectors, each thread's loads issued before its stores), then make the
+// writes visible to the tensor copies that will read them (generic -> async
+// proxy).
+__device__ __forceinline__ void stage_block_rows(const TcParams& p, int b, int kvh, int row0,
+                                                 int P, int i_lo, int i_hi, int tid) {
+  constexpr int kVec = kHeadDim * 2 / 16;   // 16-byte vectors per (token, head) row
+  constexpr int kUnroll = 4;
+  constexpr int kThreadsStage = 256;
+  const int n = (i_hi - i_lo) * kVec;
+  const uint4* srcs[2] = {static_cast<const uint4*>(p.k_new), static_cast<const uint4*>(p.v_new)};
+  uint4* dsts[2] = {static_cast<uint4*>(p.k_cache), static_cast<uint4*>(p.v_cache)};
+  for (int base = 0; base < n; base += kThreadsStage * kUnroll) {
+    uint4 v[2][kUnroll];
+    long long d[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int idx = base + u * kThreadsStage + tid;
+      d[u] = -1;
+      if (idx < n) {
+        const int i = i_lo + idx / kVec;
+        const int c = idx % kVec;
+        const int t = P + i;
+        long long tr = -1;
+        if (p.page_size == 0) {
+          tr = static_cast<long long>(b) * p.capacity + t;
+        } else {
+          const int page = p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
+          if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+          else tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+        }
+        if (tr >= 0) {
+          const long long s = (static_cast<long long>(row0 + i) * p.Hkv + kvh) * kVec + c;
+          v[0][u] = __ldg(srcs[0] + s);
+          v[1][u] = __ldg(srcs[1] + s);
+          d[u] = (tr * p.Hkv + kvh) * kVec + c;
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      if (d[u] >= 0) {
+        dsts[0][d[u]] = v[0][u];
+        dsts[1][d[u]] = v[1][u];
+      }
+    }
+  }
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  __syncwarp();
+}
+
 // One producer warp streams one of K or V through its ring.
+// With staging, the first tile that holds one of the block rows
+// [st_lo, st_hi) (relative to P) waits until the softmax warps have written
+// them.
 __device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, uint64_t* empty,
                                         int stages, uint32_t ring, const TcParams& p, Bars* bars,
                                         int b, int kvh, int t_begin, int nt, int kv_end,
-                                        int lane) {
+                                        int lane, int P, int st_lo, int st_hi) {
+  const int t_stage = st_hi > st_lo ? (P + st_lo) / kBlockN : -1;
   const bool paged = p.page_size > 0;
   const int ppt = paged ? kBlockN / p.page_size : 0;   // pages per tile
   const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
@@ -238,6 +296,10 @@ __device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, 
   bool ok = true;
   for (int i = 0; i < nt; ++i) {
     const int t = t_begin + i;
+    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p.err)) {
+      ok = false;
+      break;
+    }
     int page = -1;
     uint32_t bytes = kTileBytes;
     if (paged) {
@@ -330,6 +392,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     mbar_init(&bars->o_done[1], 1);
     mbar_init(&bars->drain, 1);
     mbar_init(&bars->kfree, 1);
+    mbar_init(&bars->staged, 8);   // every softmax warp
     bars->abort = 0;
     bars->last = 0;
   }
@@ -356,6 +419,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   const int active = (n_tiles + per_split - 1) / per_split;
   const int t_begin = split * per_split;
   const int nt = min(n_tiles, t_begin + per_split) - t_begin;
+  // Staged attention: the block rows this CTA reads, [st_lo, st_hi) relative to P.
+  int st_lo = 0, st_hi = 0;
+  if (p.k_new != nullptr && code == 0) {
+    st_lo = max(P, t_begin * kBlockN) - P;
+    st_hi = min(kv_end, (t_begin + nt) * kBlockN) - P;
+  }
 
   // The splits of a cluster merge their partials through shared memory when
   // more than one of them has keys (Sec. 5.2 step 3 split over the key range).
@@ -403,13 +472,13 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
       }
       produce(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars, b,
-              kvh, t_begin, nt, kv_end, lane);
+              kvh, t_begin, nt, kv_end, lane, P, st_lo, st_hi);
       if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
         mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
     } else if (warp == 2) {
       // ======================= V producer =======================
       produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
-              kvh, t_begin, nt, kv_end, lane);
+              kvh, t_begin, nt, kv_end, lane, P, st_lo, st_hi);
     } else if (warp == 1) {
       // ======================= MMA issuer (one elected lane) =======================
       // The whole warp walks the issue loop (waits and descriptors are
@@ -504,6 +573,13 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     float m_run = -INFINITY;  // running max, in scaled log2 units
     float l_run = 0.f;
     bool ok = true;
+
+    // Staged attention: write the block rows this CTA reads into the cache
+    // before the producers load the first tile holding one of them.
+    if (st_hi > st_lo) {
+      stage_block_rows(p, b, kvh, row0, P, st_lo, st_hi, (warp - 4) * 32 + lane);
+      if (lane == 0) mbar_arrive(&bars->staged);
+    }
 
     for (int i = 0; i < nt; ++i) {
       const int sb = i & 1;

@@ -50,6 +50,12 @@ class DeviceBatch:
                      self.n_slots, self.slot_len, self.mask_mode, self.out, self.desc,
                      self.workspace, stream=stream)
 
+    def stage_and_attend(self, stream=None) -> None:
+        """``stage`` then ``attend`` in one launch (zarya_slot_attn_staged)."""
+        zb.slot_attn_staged(self.q, self.k_new, self.v_new, self.k_cache, self.v_cache,
+                            self.cache_lens, self.page_table, self.n_slots, self.slot_len,
+                            self.mask_mode, self.out, self.desc, self.workspace, stream=stream)
+
     def commit(self, stream=None, new_lens=None) -> None:
         """Append the accepted rows and advance the lengths: in place, or into
         ``new_lens`` (leaving ``cache_lens`` as it was) when given."""

@@ -154,3 +154,16 @@ def test_commit_to_rejects_invalid_calls(lib):
     assert app(cache_lens=None) == 1
     assert app(desc=None) == 1
     assert app(k_cache=FAKE + 8) == 1
+
+
+def test_staged_rejects_missing_block_kv(lib):
+    vp = ctypes.c_void_p
+    d = _desc()
+    st = lib.zarya_slot_attn_staged(vp(FAKE), vp(None), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE),
+                                    vp(None), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE), vp(None), 0,
+                                    ctypes.byref(d), None)
+    assert st == 1
+    st = lib.zarya_slot_attn_staged(vp(FAKE), vp(FAKE), vp(FAKE + 8), vp(FAKE), vp(FAKE), vp(FAKE),
+                                    vp(None), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE), vp(None), 0,
+                                    ctypes.byref(d), None)
+    assert st == 1
