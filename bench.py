@@ -260,6 +260,12 @@ def run_ours(args):
     def attend(db):
         db.attend(stream)
 
+    def capture_fn(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn()
+        return g
+
     full, tail = divmod(K, n_rot)
     step_graph = capture(step, n_rot)
     step_tail = capture(step, tail) if tail else None
@@ -313,35 +319,74 @@ def run_ours(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         total_ms = float(t.item())
 
-    # end to end through the public API: pinned host inputs -> device, the
-    # step, output -> host, every step.
-    q_h = w.q.pin_memory()
-    kn_h = w.k_new.pin_memory()
-    vn_h = w.v_new.pin_memory()
-    acc_h = torch.as_tensor(w.accept_len).pin_memory()
-    out_h = torch.empty_like(w.q).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in (q_h, kn_h, vn_h, acc_h))
-    d2h = out_h.numel() * out_h.element_size()
+    # End to end through the public API, every step: the step's inputs (q,
+    # k_new, v_new, accept_len, packed in one pinned host buffer) copied to the
+    # device, the step, and its output copied back to pinned host memory.
+    # Copies run on their own streams, pipelined with the computation over the
+    # rotating device buffers (events order each rotation's copy-in, step and
+    # copy-out), as a serving loop would overlap transfers with compute; the
+    # n_rot steps of a rotation cycle, copies included, are one CUDA graph.
+    def align(x):
+        return (x + 255) // 256 * 256
 
-    def e2e_step(db):
-        db.q.copy_(q_h, non_blocking=True)
-        db.k_new.copy_(kn_h, non_blocking=True)
-        db.v_new.copy_(vn_h, non_blocking=True)
-        db.accept_len.copy_(acc_h, non_blocking=True)
-        step(db)
-        out_h.copy_(db.out, non_blocking=True)
+    parts = [("q", w.q), ("k_new", w.k_new), ("v_new", w.v_new),
+             ("accept_len", torch.as_tensor(w.accept_len))]
+    offs, total = [], 0
+    for _, t in parts:
+        offs.append(total)
+        total = align(total + t.numel() * t.element_size())
+    host_in = torch.zeros(total, dtype=torch.uint8).pin_memory()
+    for (_, t), o in zip(parts, offs):
+        nbytes = t.numel() * t.element_size()
+        host_in[o:o + nbytes].copy_(t.contiguous().view(-1).view(torch.uint8))
+    out_h = torch.empty_like(w.q).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for _, t in parts)
+    d2h = out_h.numel() * out_h.element_size()
+    dev_in = []
+    for db in rots:
+        buf = torch.empty(total, dtype=torch.uint8, device=dev)
+        dev_in.append(buf)
+        for (name, t), o in zip(parts, offs):
+            nbytes = t.numel() * t.element_size()
+            view = buf[o:o + nbytes].view(t.dtype).view(t.shape)
+            setattr(db, name, view)
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in rots]
+    ev_done = [torch.cuda.Event() for _ in rots]
+
+    def e2e_steps(count):
+        # stream forks off `stream` and joins back (valid inside a capture)
+        s_in.wait_stream(stream)
+        s_out.wait_stream(stream)
+        for r in range(count):
+            db = rots[r]
+            with torch.cuda.stream(s_in):
+                dev_in[r].copy_(host_in, non_blocking=True)
+                ev_in[r].record(s_in)
+            with torch.cuda.stream(stream):
+                stream.wait_event(ev_in[r])
+                step(db)
+                ev_done[r].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_done[r])
+                out_h.copy_(db.out, non_blocking=True)
+        stream.wait_stream(s_in)
+        stream.wait_stream(s_out)
 
     with torch.cuda.stream(stream):
-        for i in range(W):
-            e2e_step(rots[i % n_rot])
+        e2e_steps(n_rot)   # eager warm-up through the public API
+    torch.cuda.synchronize()
+    e2e_graph = capture_fn(lambda: e2e_steps(n_rot))
+    e2e_tail = capture_fn(lambda: e2e_steps(tail)) if tail else None
+    for _ in range(max(1, -(-W // n_rot))):
+        e2e_graph.replay()
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         e0.record(stream)
-        for i in range(K):
-            e2e_step(rots[i % n_rot])
+        run(e2e_graph, e2e_tail)
         e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
