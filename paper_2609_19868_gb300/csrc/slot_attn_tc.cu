@@ -109,6 +109,17 @@ __device__ __forceinline__ void named_bar_sync(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 
+__device__ __forceinline__ void named_bar_arrive(int id, int n) {
+  asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// Named barriers (barrier 0 is __syncthreads): 1 joins the 256 softmax
+// threads, 2-5 one quadrant's warp of each softmax group, 6 the two producer
+// warps at entry, 7 publishes the entry set-up to the other ten warps.
+constexpr int kBarSoftmax = 1;
+constexpr int kBarProducers = 6;
+constexpr int kBarSetup = 7;
+
 __device__ __forceinline__ void set_abort(Bars* bars, int* err, int code) {
   record_error(err, code);
   *reinterpret_cast<volatile int*>(&bars->abort) = 1;
@@ -281,25 +292,23 @@ __device__ __forceinline__ void stage_block_rows(const TcParams& p, int b, int k
 }
 
 // One producer warp streams one of K or V through its ring.
-// With staging, the first tile that holds one of the block rows
-// [st_lo, st_hi) (relative to P) waits until the softmax warps have written
-// them.
-__device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, uint64_t* empty,
-                                        int stages, uint32_t ring, const TcParams& p, Bars* bars,
-                                        int b, int kvh, int t_begin, int nt, int kv_end,
-                                        int lane, int P, int st_lo, int st_hi) {
-  const int t_stage = st_hi > st_lo ? (P + st_lo) / kBlockN : -1;
+// One producer warp streams one of K or V through its ring: tiles
+// [i_begin, i_end) of this CTA's range, `issued` counting the tiles whose
+// copies are in flight. With staging, the first tile that holds one of the
+// block rows [st_lo, st_hi) (relative to P) waits until the softmax warps
+// have written them. Returns false (the CTA aborts) on a bad page id or a
+// timed-out wait.
+__device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* full,
+                                              uint64_t* empty, int stages, uint32_t ring,
+                                              const TcParams& p, Bars* bars, int b, int kvh,
+                                              int t_begin, int i_begin, int i_end, int kv_end,
+                                              int lane, int t_stage, int& issued) {
   const bool paged = p.page_size > 0;
   const int ppt = paged ? kBlockN / p.page_size : 0;   // pages per tile
   const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
-  int issued = 0;
-  bool ok = true;
-  for (int i = 0; i < nt; ++i) {
+  for (int i = i_begin; i < i_end; ++i) {
     const int t = t_begin + i;
-    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p.err)) {
-      ok = false;
-      break;
-    }
+    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p.err)) return false;
     int page = -1;
     uint32_t bytes = kTileBytes;
     if (paged) {
@@ -312,8 +321,7 @@ __device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, 
       }
       if (__any_sync(0xffffffffu, bad)) {
         if (lane == 0) set_abort(bars, p.err, ZARYA_DEVERR_PAGE_ID);
-        ok = false;
-        break;
+        return false;
       }
       bytes = page_bytes * __popc(__ballot_sync(0xffffffffu, want));
     }
@@ -323,10 +331,7 @@ __device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, 
       w = wait_bar(&empty[s], ((i / stages) & 1) ^ 1, bars, p.err);
       if (w) mbar_arrive_expect_tx(&full[s], bytes);
     }
-    if (!__shfl_sync(0xffffffffu, w, 0)) {
-      ok = false;
-      break;
-    }
+    if (!__shfl_sync(0xffffffffu, w, 0)) return false;
     issued = i + 1;
     const uint32_t dst = ring + s * kTileBytes;
     if (!paged) {
@@ -340,11 +345,15 @@ __device__ __forceinline__ void produce(const CUtensorMap* map, uint64_t* full, 
       tma_load_4d(dst + kHalfBytes + o, map, &full[s], 64, kvh, 0, page);
     }
   }
-  if (!ok && lane == 0) {
-    // Let this CTA's own copies land before the CTA (and its smem) goes away.
+  return true;
+}
+
+// After a failed produce_range: let this CTA's own copies land before the CTA
+// (and its shared memory) goes away.
+__device__ __forceinline__ void drain_ring(uint64_t* full, int stages, int issued, int lane) {
+  if (lane == 0)
     for (int i = max(0, issued - stages); i < issued; ++i)
       mbar_wait(&full[i % stages], (i / stages) & 1, kDrainNs, nullptr);
-  }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -374,7 +383,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     tma_prefetch_map(&map_k);
     tma_prefetch_map(&map_v);
   }
-  if (threadIdx.x == 32) {
+  if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
     for (int s = 0; s < kStagesK; ++s) {
       mbar_init(&bars->k_full[s], 1);
@@ -395,6 +404,15 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     mbar_init(&bars->staged, 8);   // every softmax warp
     bars->abort = 0;
     bars->last = 0;
+    fence_mbar_init();
+  }
+  // The producer warps load before the CTA-wide set-up barrier (a thread
+  // with tensor copies in flight waits for them at a barrier): they only sync
+  // with each other here and arrive, without waiting, on the set-up barrier
+  // the other ten warps wait on.
+  if (warp == 0 || warp == 2) {
+    named_bar_sync(kBarProducers, 64);
+    named_bar_arrive(kBarSetup, kThreads);
   }
   // Inputs may be written by the kernel launched before this one.
   grid_dependency_wait();
@@ -441,17 +459,49 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       mbar_arrive_expect_tx(&bars->ready, cmerge_rx_bytes(n_rows_v, active, split));
     }
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = bars->tmem_base;
-  // The cluster barrier orders every CTA's barrier initialisation before any
-  // remote arrive; its wait is taken only where a thread first needs it.
-  if (p.cluster) cluster_arrive();
+  // The cluster barrier orders every CTA's barrier initialisation (released by
+  // fence.mbarrier_init) before any remote arrive; its wait is taken only
+  // where a thread first needs it. Arriving before the producers issue their
+  // first copies keeps the arrive from waiting on them.
+  if (p.cluster) cluster_arrive_relaxed();
+
+  // Producers issue Q and the first ring stages as soon as their own geometry
+  // is known (contiguous caches; stopping before a tile that waits for
+  // staging), before the CTA-wide barrier.
+  const bool works = code == 0 && r0 < R && split < active;
+  const int t_stage = st_hi > st_lo ? (P + st_lo) / kBlockN : -1;
+  int pre = 0;   // tiles issued before the barrier by each producer
+  if (works && p.page_size == 0) {
+    pre = min(nt, kStagesK);
+    if (t_stage >= 0) pre = min(pre, t_stage - t_begin);
+  }
+  int issued = 0;
+  if (warp == 0 && works) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
+      const uint32_t dq = smem_u32(smem + kOffQ);
+      tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
+      tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
+    }
+    produce_range(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars,
+                  b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
+  } else if (warp == 2 && works) {
+    produce_range(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars,
+                  b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
+  }
+
+  if (warp != 0 && warp != 2) {
+    tc_fence_before();
+    named_bar_sync(kBarSetup, kThreads);
+    tc_fence_after();
+  }
+  // TMEM base address (warp 3 wrote it before the set-up barrier); the
+  // producer warps never use it.
+  const uint32_t tmem = (warp != 0 && warp != 2) ? bars->tmem_base : 0u;
   bool cwaited = false;
   // Exits here are uniform over a cluster (its CTAs share the sequence and
   // M-tile and differ only in the split) or leave a split with no keys.
-  if (code != 0 || r0 >= R || split >= active) {
+  if (!works) {
     if (code != 0 && mt == 0 && split == 0 && threadIdx.x == 0) record_error(p.err, code);
     grid_launch_dependents();
     if (p.cluster) cluster_wait();
@@ -465,20 +515,17 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     regs_release<kRegsControl>();
     if (warp == 0) {
       // ======================= Q + K producer =======================
-      if (lane == 0) {
-        mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
-        const uint32_t dq = smem_u32(smem + kOffQ);
-        tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
-        tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
-      }
-      produce(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars, b,
-              kvh, t_begin, nt, kv_end, lane, P, st_lo, st_hi);
+      // (Q and the first `pre` K tiles were issued before the CTA barrier.)
+      if (!produce_range(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p,
+                         bars, b, kvh, t_begin, pre, nt, kv_end, lane, t_stage, issued))
+        drain_ring(bars->k_full, kStagesK, issued, lane);
       if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
         mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
     } else if (warp == 2) {
       // ======================= V producer =======================
-      produce(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars, b,
-              kvh, t_begin, nt, kv_end, lane, P, st_lo, st_hi);
+      if (!produce_range(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p,
+                         bars, b, kvh, t_begin, pre, nt, kv_end, lane, t_stage, issued))
+        drain_ring(bars->v_full, kStagesV, issued, lane);
     } else if (warp == 1) {
       // ======================= MMA issuer (one elected lane) =======================
       // The whole warp walks the issue loop (waits and descriptors are
@@ -683,7 +730,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p.err);
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_before();
-    named_bar_sync(1, 256);
+    named_bar_sync(kBarSoftmax, 256);
     tc_fence_after();
     // No Q*K^T can read Q any more: the Q buffer carries the (max, sum)
     // exchange between the groups.
@@ -691,7 +738,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     xch[m] = m_run;
     xch[128 + m] = l_run;
     tc_fence_before();
-    named_bar_sync(1, 256);
+    named_bar_sync(kBarSoftmax, 256);
     tc_fence_after();
     const float* x0 = reinterpret_cast<const float*>(smem + kOffQ);
     const float* x1 = reinterpret_cast<const float*>(smem + kOffQ + 1024);
@@ -799,14 +846,14 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         if (grp == 0) p.ws_lse[own] = lse_own;
       }
       __threadfence();
-      named_bar_sync(1, 256);
+      named_bar_sync(kBarSoftmax, 256);
       if (grp == 0 && m == 0) {
         int last = 0;
         if (*reinterpret_cast<volatile int*>(&bars->abort) == 0)
           last = (atomicAdd(&p.ws_count[unit], 1) == active - 1) ? 1 : 0;
         bars->last = last;
       }
-      named_bar_sync(1, 256);
+      named_bar_sync(kBarSoftmax, 256);
       if (*reinterpret_cast<volatile int*>(&bars->last)) {
         __threadfence();
         if (ok && row_ok) {
@@ -835,7 +882,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           }
           store_out(o, S > 0.f ? 1.f / S : 0.f);
         }
-        named_bar_sync(1, 256);
+        named_bar_sync(kBarSoftmax, 256);
         if (grp == 0 && m == 0) atomicExch(&p.ws_count[unit], 0);
       }
     }
