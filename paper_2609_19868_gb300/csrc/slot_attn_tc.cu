@@ -602,6 +602,13 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       }
     }
   } else {
+    // Staged attention: write the block rows this CTA reads into the cache
+    // before the producers load the first tile holding one of them (before
+    // the register claim, which waits for the other warpgroup's release).
+    if (st_hi > st_lo) {
+      stage_block_rows(p, b, kvh, row0, P, st_lo, st_hi, (warp - 4) * 32 + lane);
+      if (lane == 0) mbar_arrive(&bars->staged);
+    }
     regs_claim<kRegsSoftmax>();
     // ======================= softmax + epilogue =======================
     // Both groups work on every key tile: group g takes its keys
@@ -621,12 +628,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     float l_run = 0.f;
     bool ok = true;
 
-    // Staged attention: write the block rows this CTA reads into the cache
-    // before the producers load the first tile holding one of them.
-    if (st_hi > st_lo) {
-      stage_block_rows(p, b, kvh, row0, P, st_lo, st_hi, (warp - 4) * 32 + lane);
-      if (lane == 0) mbar_arrive(&bars->staged);
-    }
 
     for (int i = 0; i < nt; ++i) {
       const int sb = i & 1;
