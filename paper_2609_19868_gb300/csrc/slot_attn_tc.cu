@@ -726,21 +726,13 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     }
 
     // ---- epilogue: merge the two groups' partial results per row ----
-    // The last P*V completes after every other MMA of the CTA; P*V(nt-3) is
-    // known complete, so the parity wait cannot alias an older phase.
-    if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p.err);
-    ok = __all_sync(0xffffffffu, ok);
-    tc_fence_before();
-    named_bar_sync(kBarSoftmax, 256);
-    tc_fence_after();
-    // No Q*K^T can read Q any more: the Q buffer carries the (max, sum)
-    // exchange between the groups.
+    // Each group has seen the last S, so no Q*K^T reads Q any more: the Q
+    // buffer carries the (max, sum) exchange between the groups, done while
+    // the last P*V still runs.
     float* xch = reinterpret_cast<float*>(smem + kOffQ + grp * 1024);
     xch[m] = m_run;
     xch[128 + m] = l_run;
-    tc_fence_before();
     named_bar_sync(kBarSoftmax, 256);
-    tc_fence_after();
     const float* x0 = reinterpret_cast<const float*>(smem + kOffQ);
     const float* x1 = reinterpret_cast<const float*>(smem + kOffQ + 1024);
     const float mA = x0[m], lA = x0[128 + m];
@@ -754,6 +746,11 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     const long long unit = static_cast<long long>(bh) * p.m_tiles + mt;
     const int col0 = grp * 64;   // group g finishes columns [64g, 64g + 64)
     grid_launch_dependents();
+    // The last P*V completes after every other MMA of the CTA; P*V(nt-3) is
+    // known complete, so the parity wait cannot alias an older phase.
+    if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p.err);
+    ok = __all_sync(0xffffffffu, ok);
+    tc_fence_after();
 
     // This CTA's result for its 64 columns of row m, normalised.
     float o[64];
