@@ -69,18 +69,6 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
-// ---------------------------------------------------------------- registers
-// Per-warpgroup register budget (all four warps of a warpgroup execute it).
-template <int kRegs>
-__device__ __forceinline__ void regs_release() {
-  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegs));
-}
-
-template <int kRegs>
-__device__ __forceinline__ void regs_claim() {
-  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegs));
-}
-
 // ---------------------------------------------------------------- PDL
 // Programmatic dependent launch: wait until the grids this one depends on have
 // completed and their writes are visible (a no-op when launched without the

@@ -61,11 +61,6 @@ constexpr uint32_t kOffV = kOffK + kStagesK * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStagesV * kTileBytes;
 constexpr uint32_t kTmemCols = 512;  // S0/P0 [0,128) S1/P1 [128,256) O0 [256,384) O1 [384,512)
 constexpr uint32_t kTmemO = 256;
-constexpr int kRegsLaunch = 168;    // 65536 / 384, rounded down to a multiple of 8
-constexpr int kRegsControl = 64;    // warps 0-3
-constexpr int kRegsSoftmax = 216;   // warps 4-11
-static_assert(4 * 32 * kRegsControl + 8 * 32 * kRegsSoftmax <= kThreads * kRegsLaunch,
-              "register split exceeds the launch allocation");
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
 constexpr uint64_t kDrainNs = 100000000ull;  // 100 ms
 
@@ -238,65 +233,68 @@ __device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity,
   return false;
 }
 
-// Staged attention: copy block rows [i_lo, i_hi) of sequence b, KV head kvh,
-// of K and V from k_new / v_new ([total_rows, Hkv, D]) to cache positions
-// P + i (the 256 softmax threads, idle until the first S tile; 16-byte
-// vectors, each thread's loads issued before its stores), then make the
-// writes visible to the tensor copies that will read them (generic -> async
-// proxy).
-__device__ __forceinline__ void stage_block_rows(const TcParams& p, int b, int kvh, int row0,
-                                                 int P, int i_lo, int i_hi, int tid) {
-  constexpr int kVec = kHeadDim * 2 / 16;   // 16-byte vectors per (token, head) row
-  constexpr int kUnroll = 4;
-  constexpr int kThreadsStage = 256;
-  const int n = (i_hi - i_lo) * kVec;
-  const uint4* srcs[2] = {static_cast<const uint4*>(p.k_new), static_cast<const uint4*>(p.v_new)};
-  uint4* dsts[2] = {static_cast<uint4*>(p.k_cache), static_cast<uint4*>(p.v_cache)};
-  for (int base = 0; base < n; base += kThreadsStage * kUnroll) {
-    uint4 v[2][kUnroll];
-    long long d[kUnroll];
+// Staged attention: warp 3 (idle until the merge) copies the block rows
+// [i_lo, i_hi) of sequence b, KV head kvh, of K and V from k_new / v_new
+// ([total_rows, Hkv, D]) to cache positions P + i, with kRound 16-byte
+// vectors of each tensor per lane in flight per round, then fences the writes
+// against the async proxy; the producers wait on `staged` before loading the
+// first tile that holds one of these rows.
+struct WarpStager {
+  static constexpr int kVec = kHeadDim * 2 / 16;   // 16-byte vectors per (token, head) row
+  static constexpr int kRound = 12;
+
+  __device__ __forceinline__ static void run(const TcParams& p, int b, int kvh, int row0, int P,
+                                             int i_lo, int i_hi, int lane) {
+    const uint4* kn = static_cast<const uint4*>(p.k_new);
+    const uint4* vn = static_cast<const uint4*>(p.v_new);
+    uint4* kc = static_cast<uint4*>(p.k_cache);
+    uint4* vc = static_cast<uint4*>(p.v_cache);
+    const int n = (i_hi - i_lo) * kVec;
+    for (int base = 0; base < n; base += kRound * 32) {
+      uint4 vk[kRound], vv[kRound];
+      long long d[kRound];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int idx = base + u * kThreadsStage + tid;
-      d[u] = -1;
-      if (idx < n) {
-        const int i = i_lo + idx / kVec;
-        const int c = idx % kVec;
-        const int t = P + i;
-        long long tr = -1;
-        if (p.page_size == 0) {
-          tr = static_cast<long long>(b) * p.capacity + t;
-        } else {
-          const int page = p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
-          if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
-          else tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+      for (int u = 0; u < kRound; ++u) {
+        const int idx = base + u * 32 + lane;
+        d[u] = -1;
+        if (idx < n) {
+          const int i = i_lo + idx / kVec;
+          const int c = idx % kVec;
+          const int t = P + i;
+          long long tr = -1;
+          if (p.page_size == 0) {
+            tr = static_cast<long long>(b) * p.capacity + t;
+          } else {
+            const int page =
+                p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
+            if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+            else tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
+          }
+          if (tr >= 0) {
+            const long long sidx = (static_cast<long long>(row0 + i) * p.Hkv + kvh) * kVec + c;
+            vk[u] = __ldg(kn + sidx);
+            vv[u] = __ldg(vn + sidx);
+            d[u] = (tr * p.Hkv + kvh) * kVec + c;
+          }
         }
-        if (tr >= 0) {
-          const long long s = (static_cast<long long>(row0 + i) * p.Hkv + kvh) * kVec + c;
-          v[0][u] = __ldg(srcs[0] + s);
-          v[1][u] = __ldg(srcs[1] + s);
-          d[u] = (tr * p.Hkv + kvh) * kVec + c;
+      }
+#pragma unroll
+      for (int u = 0; u < kRound; ++u) {
+        if (d[u] >= 0) {
+          kc[d[u]] = vk[u];
+          vc[d[u]] = vv[u];
         }
       }
     }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      if (d[u] >= 0) {
-        dsts[0][d[u]] = v[0][u];
-        dsts[1][d[u]] = v[1][u];
-      }
-    }
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    __syncwarp();
   }
-  asm volatile("fence.proxy.async.global;" ::: "memory");
-  __syncwarp();
-}
+};
 
 // One producer warp streams one of K or V through its ring.
 // One producer warp streams one of K or V through its ring: tiles
 // [i_begin, i_end) of this CTA's range, `issued` counting the tiles whose
-// copies are in flight. With staging, the first tile that holds one of the
-// block rows [st_lo, st_hi) (relative to P) waits until the softmax warps
-// have written them. Returns false (the CTA aborts) on a bad page id or a
+// copies are in flight. Returns false (the CTA aborts) on a bad page id or a
 // timed-out wait.
 __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* full,
                                               uint64_t* empty, int stages, uint32_t ring,
@@ -401,7 +399,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     mbar_init(&bars->o_done[1], 1);
     mbar_init(&bars->drain, 1);
     mbar_init(&bars->kfree, 1);
-    mbar_init(&bars->staged, 8);   // every softmax warp
+    mbar_init(&bars->staged, 1);
     bars->abort = 0;
     bars->last = 0;
     fence_mbar_init();
@@ -466,8 +464,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   if (p.cluster) cluster_arrive_relaxed();
 
   // Producers issue Q and the first ring stages as soon as their own geometry
-  // is known (contiguous caches; stopping before a tile that waits for
-  // staging), before the CTA-wide barrier.
+  // is known (contiguous caches; stopping before a tile that holds a staged
+  // block row), before the CTA-wide barrier.
   const bool works = code == 0 && r0 < R && split < active;
   const int t_stage = st_hi > st_lo ? (P + st_lo) / kBlockN : -1;
   int pre = 0;   // tiles issued before the barrier by each producer
@@ -476,18 +474,21 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     if (t_stage >= 0) pre = min(pre, t_stage - t_begin);
   }
   int issued = 0;
-  if (warp == 0 && works) {
-    if (lane == 0) {
-      mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
-      const uint32_t dq = smem_u32(smem + kOffQ);
-      tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
-      tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
+  if ((warp == 0 || warp == 2) && works) {
+    const bool is_k = warp == 0;
+    if (is_k) {
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bars->q_full, kTileBytes);
+        const uint32_t dq = smem_u32(smem + kOffQ);
+        tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0);
+        tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0);
+      }
+      produce_range(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p,
+                    bars, b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
+    } else {
+      produce_range(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p,
+                    bars, b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
     }
-    produce_range(&map_k, bars->k_full, bars->k_empty, kStagesK, smem_u32(smem + kOffK), p, bars,
-                  b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
-  } else if (warp == 2 && works) {
-    produce_range(&map_v, bars->v_full, bars->v_empty, kStagesV, smem_u32(smem + kOffV), p, bars,
-                  b, kvh, t_begin, 0, pre, kv_end, lane, t_stage, issued);
   }
 
   if (warp != 0 && warp != 2) {
@@ -509,10 +510,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     return;
   }
 
-  // Registers: the producer / MMA / TMEM warpgroup hands most of its share to
-  // the two softmax warpgroups (128 x 64 + 256 x 216 <= 384 x 168 at launch).
   if (warp < 4) {
-    regs_release<kRegsControl>();
     if (warp == 0) {
       // ======================= Q + K producer =======================
       // (Q and the first `pre` K tiles were issued before the CTA barrier.)
@@ -589,6 +587,11 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
       }
     } else if (warp == 3) {
+      // ======================= staging of the block's own K/V =======================
+      if (st_hi > st_lo) {
+        WarpStager::run(p, b, kvh, row0, P, st_lo, st_hi, lane);
+        if (lane == 0) mbar_arrive(&bars->staged);
+      }
       // ======================= cluster merge: K ring hand-off =======================
       // Once this CTA's last Q*K^T has completed no copy or MMA touches its K
       // ring again: tell the other splits they may write their rows into it.
@@ -602,14 +605,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       }
     }
   } else {
-    // Staged attention: write the block rows this CTA reads into the cache
-    // before the producers load the first tile holding one of them (before
-    // the register claim, which waits for the other warpgroup's release).
-    if (st_hi > st_lo) {
-      stage_block_rows(p, b, kvh, row0, P, st_lo, st_hi, (warp - 4) * 32 + lane);
-      if (lane == 0) mbar_arrive(&bars->staged);
-    }
-    regs_claim<kRegsSoftmax>();
     // ======================= softmax + epilogue =======================
     // Both groups work on every key tile: group g takes its keys
     // [64g, 64g + 64) with a running max / sum of its own and accumulates
