@@ -187,6 +187,25 @@ def dist_setup():
     return world, rank, local
 
 
+def max_over_ranks(x: float, device, world: int) -> float:
+    """The maximum of a per-rank time over all ranks: the slowest replica
+    sets the job's time (a no-op on one rank)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(steps: int, world: int, total_ms: float) -> float:
+    """Whole-job steps/s of `world` replicas that each ran `steps` steps, the
+    slowest taking total_ms (weak scaling: every rank has its own batch)."""
+    return steps * world / (total_ms * 1e-3)
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -311,13 +330,10 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = sampler.stop(t0, time.time()) if sampler else None
     assert zb.check_device_error(stream) == 0
-    attn_ms = a0.elapsed_time(a1) / K
+    attn_ms = max_over_ranks(a0.elapsed_time(a1) / K, dev, world)
     attn_method = (f"{K} attention launches back to back ({n_rot} per CUDA graph, one per cache "
                    "rotation), CUDA events on the launching stream")
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev, world)
 
     # End to end through the public API, every step: the step's inputs (q,
     # k_new, v_new, accept_len, packed in one pinned host buffer) copied to the
@@ -390,16 +406,13 @@ def run_ours(args):
         e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e2e_ms, dev, world)
     assert zb.check_device_error(stream) == 0
 
     hbm_peak, tf_peak, peak_src = read_peaks()
     attn_gbs = counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9
     attn_tflops = counts["flops"] / (attn_ms * 1e-3) / 1e12
-    value = K * world / (total_ms * 1e-3)
+    value = replica_throughput(K, world, total_ms)
     line = {
         "metric": "slot-decode steps/s (one layer: stage + slot attention + commit)",
         "value": round(value, 2),
@@ -434,7 +447,7 @@ def run_ours(args):
         "roofline": roofline_entry(counts, attn_gbs, attn_tflops, hbm_peak, tf_peak, peak_src,
                                    recorded_traffic(args.workload)),
         "e2e": {
-            "value": round(K * world / (e2e_ms * 1e-3), 2),
+            "value": round(replica_throughput(K, world, e2e_ms), 2),
             "unit": "steps/s",
             "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h),
