@@ -20,6 +20,9 @@ Mask modes (Sec. 5.2):
      and the whole block;
   1  slot-causal (verification pass, step 6): block row r sees the prefix and
      block rows 0..r, i.e. plain causal attention over the reordered sequence.
+  2  slot-independent (step 6 for several selected slots at once, each
+     verified on its own): block row r = s*L + j sees the prefix and rows
+     s*L .. r of its own slot.
 """
 from __future__ import annotations
 
@@ -35,6 +38,7 @@ _SRC = os.path.join(_HERE, "slot_attn_oracle.c")
 
 MODE_BIDIR_BLOCK = 0
 MODE_SLOT_CAUSAL = 1
+MODE_SLOT_INDEPENDENT = 2
 
 _F64, _F32, _BF16 = 0, 1, 2
 
@@ -202,8 +206,9 @@ def slot_attn_dense(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_l
                     q_row_offsets=None, *, scale: float, page_size: int = 0) -> np.ndarray:
     """Brute force: per sequence, build the square mask of the reordered
     sequence [prefix ; block] (all-ones for mode 0's block rows, lower
-    triangular for mode 1), take the block's rows, and apply it to the full
-    score matrix. fp64 throughout."""
+    triangular for mode 1, block-diagonal lower triangular over the slots for
+    mode 2), take the block's rows, and apply it to the full score matrix.
+    fp64 throughout."""
     q = _as_numpy(q)
     lens = np.asarray(_as_numpy(cache_lens), dtype=np.int64)
     ns = np.asarray(_as_numpy(n_slots), dtype=np.int64)
@@ -229,6 +234,12 @@ def slot_attn_dense(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_l
             full = np.tril(np.ones((n, n), dtype=bool))
         elif mm[b] == MODE_BIDIR_BLOCK:
             full = np.ones((n, n), dtype=bool)
+        elif mm[b] == MODE_SLOT_INDEPENDENT:
+            full = np.tril(np.ones((n, n), dtype=bool))
+            L = int(sl[b])
+            slot = np.arange(R) // L            # slot of each block position
+            same = slot[:, None] == slot[None, :]
+            full[P:, P:] &= same                # no key of another slot
         else:
             raise ValueError("bad mask mode")
         mask = full[P:P + R]  # block rows of the reordered sequence

@@ -21,6 +21,10 @@
  *       c < P_b + R_b
  *     mode 1 (slot-causal, verification / AR infilling, step 6):
  *       c < P_b + r + 1   (causal over the reordered, flattened sequence)
+ *     mode 2 (slot-independent verification: each selected slot verified on
+ *       its own, step 6 run for several slots in one pass), for row
+ *       r = s * L_b + j (slot s, offset j):
+ *       c < P_b  or  P_b + s * L_b <= c <= P_b + r
  *
  * Every value is read exactly (bf16 / fp32 -> fp64 is exact) and every sum is
  * taken in fp64 in key order. No tiling, no online softmax, no splitting.
@@ -92,14 +96,18 @@ static int attend_one(const or_problem* p, int b, int h, int r, int64_t n_pages,
   const int64_t P = p->cache_lens[b];
   const int64_t R = (int64_t)p->n_slots[b] * p->slot_len[b];
   if (r < 0 || r >= R) return -1;
-  int64_t n_vis;
-  if (p->mask_mode[b] == 0) n_vis = P + R;
-  else if (p->mask_mode[b] == 1) n_vis = P + r + 1;
-  else return -1;
+  const int mode = p->mask_mode[b];
+  if (mode < 0 || mode > 2) return -1;
+  /* keys beyond the last visible one are never read */
+  const int64_t n_vis = (mode == 0) ? P + R : P + r + 1;
+  /* mode 2 also hides the block rows of the earlier slots: [P, P + s * L) */
+  const int64_t L = p->slot_len[b];
+  const int64_t hide_lo = P, hide_hi = (mode == 2) ? P + (r / L) * L : P;
 
   const int64_t qbase = ((p->q_row_offsets[b] + r) * p->Hq + h) * (int64_t)p->D;
   double m = -INFINITY;
   for (int64_t c = 0; c < n_vis; ++c) {
+    if (c >= hide_lo && c < hide_hi) continue;
     const int64_t kb = kv_index(p, b, c, j, n_pages);
     if (kb < 0) return -1;
     double dot = 0.0;
@@ -111,6 +119,7 @@ static int attend_one(const or_problem* p, int b, int h, int r, int64_t n_pages,
   double denom = 0.0;
   for (int d = 0; d < p->D; ++d) out[d] = 0.0;
   for (int64_t c = 0; c < n_vis; ++c) {
+    if (c >= hide_lo && c < hide_hi) continue;
     const double w = exp(sigma[c] - m);
     denom += w;
     const int64_t vb = kv_index(p, b, c, j, n_pages);

@@ -79,17 +79,17 @@ def sdpa(q, k, v, scale, causal, gqa=False):
 # ---------------------------------------------------------------- brute force
 
 def test_c_matches_dense_bruteforce_exhaustive(oracle_mod):
-    """Every S*L <= 8, P in 0..4, both modes, contiguous and paged, two
+    """Every S*L <= 8, P in 0..4, the three modes, contiguous and paged, two
     sequences with different prefixes: C oracle == dense-mask brute force."""
     rng = np.random.default_rng(100)
     shapes = [(s, l) for s in (1, 2, 4, 8) for l in (1, 2, 4, 8) if s * l <= 8]
     n = 0
     for S, L in shapes:
         for P in range(5):
-            for mode in (0, 1):
+            for mode in (0, 1, 2):
                 for page_size in (0, 2):
                     pb = make_problem(rng, [P, (P + 3) % 5], [S, S], [L, max(1, L // 2)],
-                                      [mode, 1 - mode], page_size=page_size)
+                                      [mode, (mode + 1) % 3], page_size=page_size)
                     got = run_c(oracle_mod, pb, 0.37)
                     ref = oracle_mod.slot_attn_dense(
                         pb["q"], pb["k_cache"], pb["v_cache"], pb["cache_lens"],
@@ -97,7 +97,7 @@ def test_c_matches_dense_bruteforce_exhaustive(oracle_mod):
                         pb["q_row_offsets"], scale=0.37, page_size=page_size)
                     np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
                     n += 1
-    assert n == len(shapes) * 5 * 2 * 2
+    assert n == len(shapes) * 5 * 3 * 2
 
 
 # ---------------------------------------------------------------- library pins
@@ -122,6 +122,39 @@ def test_slot_causal_equals_textbook_causal_attention(oracle_mod, P, S, L):
     vfull = pb["seqs_v"][0].transpose(1, 0, 2).copy()
     ref = sdpa(qfull, kfull, vfull, 0.25, causal=True)[:, P:n].transpose(1, 0, 2)
     np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("P,S,L", [(0, 3, 1), (6, 4, 2), (11, 3, 5), (4, 2, 8)])
+def test_slot_independent_equals_each_slot_verified_alone(oracle_mod, P, S, L):
+    """Slot-independent rows of slot s == the last L rows of plain causal
+    attention computed from scratch over [prefix; slot s's tokens] alone: the
+    S selected slots are verified in one pass exactly as S separate
+    verification passes would (Sec. 5.2 step 6). torch SDPA is the reference;
+    with L = 1 each row sees the prefix and itself."""
+    rng = np.random.default_rng(900 + P * 13 + S * 5 + L)
+    Hq = Hkv = 2
+    D = 16
+    pb = make_problem(rng, [P], [S], [L], [2], Hq=Hq, Hkv=Hkv, D=D)
+    got = run_c(oracle_mod, pb, 0.3)
+    q_prefix = rng.standard_normal((P, Hq, D))
+    k_all, v_all = pb["seqs_k"][0], pb["seqs_v"][0]
+    for s_ in range(S):
+        rows = slice(s_ * L, (s_ + 1) * L)
+        keys = np.r_[np.arange(P), P + np.arange(s_ * L, (s_ + 1) * L)]
+        qfull = np.concatenate([q_prefix, pb["q"][rows]]).transpose(1, 0, 2).copy()
+        kfull = k_all[keys].transpose(1, 0, 2).copy()
+        vfull = v_all[keys].transpose(1, 0, 2).copy()
+        ref = sdpa(qfull, kfull, vfull, 0.3, causal=True)[:, P:].transpose(1, 0, 2)
+        np.testing.assert_allclose(got[rows], ref, rtol=0, atol=1e-12)
+
+
+def test_slot_independent_with_one_slot_is_slot_causal(oracle_mod):
+    rng = np.random.default_rng(77)
+    pb = make_problem(rng, [9, 0], [1, 1], [6, 5], [2, 2])
+    got = run_c(oracle_mod, pb, 0.4)
+    pb["mask_mode"] = np.asarray([1, 1], dtype=np.int32)
+    ref = run_c(oracle_mod, pb, 0.4)
+    np.testing.assert_array_equal(got, ref)
 
 
 @pytest.mark.parametrize("P", [0, 1, 6, 40])
@@ -332,7 +365,7 @@ def test_rejects_bad_page_ids_and_modes(oracle_mod):
     pb["page_table"][0, 1] = pb["n_pages"] + 5
     with pytest.raises(ValueError):
         run_c(oracle_mod, pb, 0.3)
-    pb = make_problem(rng, [7], [2], [4], [2])
+    pb = make_problem(rng, [7], [2], [4], [3])
     with pytest.raises(ValueError):
         run_c(oracle_mod, pb, 0.3)
 
