@@ -57,7 +57,12 @@ typedef enum {
   ZARYA_MASK_BIDIR_BLOCK = 0,
   /* Verification pass (step 6, intra-slot autoregressive infilling): causal
    * over the reordered, flattened sequence: visible(c) <=> c < P_b + r + 1. */
-  ZARYA_MASK_SLOT_CAUSAL = 1
+  ZARYA_MASK_SLOT_CAUSAL = 1,
+  /* Verification of several selected slots in one pass, each on its own
+   * (step 6 with parallel slots): block row r = s*L_b + j sees the prefix and
+   * rows s*L_b .. r of its own slot:
+   * visible(c) <=> c < P_b or P_b + s*L_b <= c <= P_b + r. */
+  ZARYA_MASK_SLOT_INDEPENDENT = 2
 } zarya_mask_mode;
 
 typedef enum { ZARYA_BF16 = 0, ZARYA_FP32 = 1 } zarya_dtype;

@@ -43,7 +43,9 @@ namespace {
 __device__ __forceinline__ int check_sequence(const SimtParams& p, int b, int* P_out, int* R_out,
                                               int* mode_out, int* row0_out) {
   const int P = p.cache_lens[b];
-  const int R = p.n_slots[b] * p.slot_len[b];
+  // R_b = S_b * L_b, clamped so that an absurd product reads as invalid below
+  const long long R64 = static_cast<long long>(p.n_slots[b]) * p.slot_len[b];
+  const int R = R64 > p.max_rows ? p.max_rows + 1 : static_cast<int>(R64);
   const int mode = p.mask_mode[b];
   const int row0 = p.q_row_offsets[b];
   const int row_end = p.q_row_offsets[b + 1];
@@ -51,8 +53,11 @@ __device__ __forceinline__ int check_sequence(const SimtParams& p, int b, int* P
   *R_out = R;
   *mode_out = mode;
   *row0_out = row0;
-  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL) return ZARYA_DEVERR_MASK_MODE;
-  if (R <= 0 || R > p.max_rows || row_end - row0 != R || row0 < 0 || row_end > p.total_rows)
+  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL &&
+      mode != ZARYA_MASK_SLOT_INDEPENDENT)
+    return ZARYA_DEVERR_MASK_MODE;
+  if (p.n_slots[b] < 1 || p.slot_len[b] < 1 || R > p.max_rows || row_end - row0 != R ||
+      row0 < 0 || row_end > p.total_rows)
     return ZARYA_DEVERR_ROWS;
   if (P < 0 || static_cast<long long>(P) + R > p.capacity) return ZARYA_DEVERR_CAPACITY;
   return 0;
@@ -93,6 +98,8 @@ slot_attn_f32_kernel(const SimtParams p) {
   const int g = p.Hq / p.Hkv;
   const int j = h / g;
   const int n_vis = (mode == ZARYA_MASK_BIDIR_BLOCK) ? P + R : P + r + 1;
+  // slot-independent: the earlier slots' block rows [P, P + s L) are hidden
+  const int hide_hi = (mode == ZARYA_MASK_SLOT_INDEPENDENT) ? P + (r / p.slot_len[b]) * p.slot_len[b] : P;
   const float* q = reinterpret_cast<const float*>(p.q) +
                    (static_cast<long long>(row0 + r) * p.Hq + h) * D;
   const float* kc = reinterpret_cast<const float*>(p.k_cache);
@@ -105,6 +112,7 @@ slot_attn_f32_kernel(const SimtParams p) {
   }
   float m = -INFINITY, l = 0.f;
   for (int c = 0; c < n_vis; ++c) {
+    if (c == P && hide_hi > P) c = hide_hi;   // skip the hidden block rows
     const long long tr =
         token_row(p.page_table, p.page_size, p.max_pages, p.n_pages, p.capacity, b, c);
     if (tr < 0) {

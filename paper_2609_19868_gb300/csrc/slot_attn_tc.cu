@@ -417,19 +417,24 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
 
   // ---- per-sequence geometry (uniform over the CTA) ----
   const int P = p.cache_lens[b];
-  const int R = p.n_slots[b] * p.slot_len[b];
+  // R_b = S_b * L_b, clamped so that an absurd product reads as invalid below
+  const long long R64 = static_cast<long long>(p.n_slots[b]) * p.slot_len[b];
+  const int R = R64 > p.max_rows ? p.max_rows + 1 : static_cast<int>(R64);
   const int mode = p.mask_mode[b];
   const int row0 = p.q_row_offsets[b];
   const int row_end = p.q_row_offsets[b + 1];
   int code = 0;
-  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL) code = ZARYA_DEVERR_MASK_MODE;
-  else if (R <= 0 || R > p.max_rows || row_end - row0 != R || row0 < 0 || row_end > p.total_rows)
+  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL &&
+      mode != ZARYA_MASK_SLOT_INDEPENDENT)
+    code = ZARYA_DEVERR_MASK_MODE;
+  else if (p.n_slots[b] < 1 || p.slot_len[b] < 1 || R > p.max_rows || row_end - row0 != R ||
+           row0 < 0 || row_end > p.total_rows)
     code = ZARYA_DEVERR_ROWS;
   else if (P < 0 || static_cast<long long>(P) + R > p.capacity) code = ZARYA_DEVERR_CAPACITY;
   const int rows_per_tile = kBlockM / p.g;
   const int r0 = mt * rows_per_tile;
   const int r_hi = min(r0 + rows_per_tile, R) - 1;
-  const int kv_end = (mode == ZARYA_MASK_SLOT_CAUSAL) ? P + r_hi + 1 : P + R;
+  const int kv_end = (mode == ZARYA_MASK_BIDIR_BLOCK) ? P + R : P + r_hi + 1;
   const int n_tiles = (code != 0 || kv_end <= 0) ? 1 : (kv_end + kBlockN - 1) / kBlockN;
   const int per_split = max(1, (n_tiles + p.splits - 1) / p.splits);
   const int active = (n_tiles + per_split - 1) / per_split;
@@ -615,7 +620,10 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     const int r = r0 + m / p.g;
     const int h = kvh * p.g + (m - (m / p.g) * p.g);
     const bool row_ok = r <= r_hi;
-    const int limit = !row_ok ? kv_end : (mode == ZARYA_MASK_SLOT_CAUSAL ? P + r + 1 : P + R);
+    const int limit = !row_ok ? kv_end : (mode == ZARYA_MASK_BIDIR_BLOCK ? P + R : P + r + 1);
+    // slot-independent: the block rows of the earlier slots, [P, hide_hi)
+    const int hide_hi =
+        (row_ok && mode == ZARYA_MASK_SLOT_INDEPENDENT) ? P + (r / p.slot_len[b]) * p.slot_len[b] : P;
     const uint32_t t_row = tmem + (static_cast<uint32_t>(wq * 32) << 16);
     const uint32_t t_o = t_row + kTmemO + grp * 128;
     const float sl2 = p.scale_log2;
@@ -638,6 +646,11 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
 #pragma unroll
         for (int x = 0; x < 64; ++x)
           if (c0 + x >= limit) s[x] = -INFINITY;
+      }
+      if (hide_hi > P && c0 < hide_hi && c0 + 64 > P) {
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+          if (c0 + x >= P && c0 + x < hide_hi) s[x] = -INFINITY;
       }
       float mx[8];
 #pragma unroll
