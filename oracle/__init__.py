@@ -14,6 +14,9 @@ Three independent formulations live here:
   score matrix; used to pin the C code on tiny shapes.
 * ``kv_append``: the cache update with accepted tokens (Sec. 5.2 step 7) as a
   plain row copy in numpy.
+* ``oracle.sampling``: slot selection and token acceptance (Sec. 5.2 steps
+  3-6): draws, Gumbel-max sampling, slot confidences, the selection rule and
+  the accepted prefixes, in numpy fp64.
 
 Mask modes (Sec. 5.2):
   0  block-bidirectional (draft pass, step 3): block rows see the whole prefix
