@@ -193,18 +193,22 @@ def _offsets(row_offsets, n_slots, slot_len):
 def draft_select(logits, n_slots, slot_len, *, temperature: float, slot_threshold: float,
                  seed: int = 0, offset: int = 0, row_offsets=None, max_slots=None,
                  rows=None, fast: bool = False):
-    """Steps 3-5 for a batch. ``logits`` is [total_rows, V] (any float type,
-    read as fp64; bf16 callers pass the values widened to float32), with
-    sequence b's block in rows row_offsets[b] .. row_offsets[b] + S_b L_b,
-    slot s in rows s L_b .. s L_b + L_b - 1 of it.
+    """Steps 3-5 for a batch. ``logits`` is [total_rows, V] (read as fp64;
+    bf16 callers pass the values widened to float32). Sequence b's block is
+    rows row_offsets[b] .. row_offsets[b] + S_b L_b - 1 (default offsets: the
+    running sum of S_b L_b), slot s in its rows s L_b .. s L_b + L_b - 1.
 
     Returns a dict with
-      draft_tokens [total_rows] int32, draft_prob [total_rows] float64,
+      draft_tokens [total_rows] int32 and draft_prob [total_rows] float64
+        (-1 / NaN on rows outside every block),
       slot_conf [B, max_slots] (0 past S_b), slot_selected [B, max_slots] uint8,
       n_selected [B] int32,
-      verify_rows [total_rows] int32: in sequence b's segment, the block-row
-        indices of the selected slots' rows in slot order, then -1,
-      verify_tokens [total_rows] int32: the drafted tokens of those rows, -1 after.
+      verify_row_offsets [B + 1] int64: the verification block's layout, the
+        running sum of n_selected_b L_b (its rows are packed densely),
+      verify_src_rows [total_rows] int32: for verification row
+        verify_row_offsets[b] + k, the global draft row it verifies (the
+        selected slots' rows in slot order); -1 from verify_row_offsets[B] on,
+      verify_tokens [total_rows] int32: the tokens drafted at those rows, -1 after.
     ``rows``, if given, restricts the per-row draw to those global rows (the
     other entries stay -1 / NaN and selection is skipped): for sampled checks
     of full-size workloads."""
@@ -217,10 +221,10 @@ def draft_select(logits, n_slots, slot_len, *, temperature: float, slot_threshol
     draw = _draw_token_fast if fast else draw_token
     tokens = np.full(total, -1, dtype=np.int32)
     prob = np.full(total, np.nan)
-    todo = range(total) if rows is None else [int(r) for r in rows]
     active = np.zeros(total, dtype=bool)
     for b in range(B):
         active[offs[b]: offs[b] + ns[b] * sl[b]] = True
+    todo = range(total) if rows is None else [int(r) for r in rows]
     for g in todo:
         if not active[g]:
             continue
@@ -234,7 +238,8 @@ def draft_select(logits, n_slots, slot_len, *, temperature: float, slot_threshol
     conf = np.zeros((B, max_slots))
     sel = np.zeros((B, max_slots), dtype=np.uint8)
     n_sel = np.zeros(B, dtype=np.int32)
-    vrows = np.full(total, -1, dtype=np.int32)
+    voffs = np.zeros(B + 1, dtype=np.int64)
+    src = np.full(total, -1, dtype=np.int32)
     vtok = np.full(total, -1, dtype=np.int32)
     for b in range(B):
         S, L, o = int(ns[b]), int(sl[b]), int(offs[b])
@@ -243,44 +248,39 @@ def draft_select(logits, n_slots, slot_len, *, temperature: float, slot_threshol
         mask = select_slots(c, slot_threshold)
         sel[b, :S] = mask
         n_sel[b] = int(mask.sum())
-        k = 0
+        voffs[b + 1] = voffs[b] + n_sel[b] * L
+        k = int(voffs[b])
         for s in range(S):
             if mask[s]:
                 for j in range(L):
-                    vrows[o + k] = s * L + j
-                    vtok[o + k] = tokens[o + s * L + j]
+                    src[k] = o + s * L + j
+                    vtok[k] = tokens[o + s * L + j]
                     k += 1
-    out.update(slot_conf=conf, slot_selected=sel, n_selected=n_sel, verify_rows=vrows,
-               verify_tokens=vtok)
+    out.update(slot_conf=conf, slot_selected=sel, n_selected=n_sel, verify_row_offsets=voffs,
+               verify_src_rows=src, verify_tokens=vtok)
     return out
 
 
-def verify_accept(logits, tokens, n_selected, slot_len, *, temperature: float,
-                  token_threshold: float, row_offsets=None, n_slots=None, max_slots=None,
-                  rows=None):
-    """Step 6 for a batch. Verification row k of sequence b (k < n_sel_b L_b)
-    is global row row_offsets[b] + k of ``logits`` and carries token
-    ``tokens[row_offsets[b] + k]``. ``row_offsets`` defaults to the draft
-    layout S_b L_b (``n_slots``) or, without it, to n_sel_b L_b.
+def verify_accept(logits, tokens, n_slots, slot_len, *, temperature: float,
+                  token_threshold: float, row_offsets=None, max_slots=None, rows=None):
+    """Step 6 for a batch. ``n_slots[b]`` is the number of slots verified for
+    sequence b (n_selected of the draft) and its verification rows are
+    row_offsets[b] .. row_offsets[b] + n_slots[b] L_b - 1 of ``logits``
+    (default: packed densely), row k carrying token ``tokens[row]``.
 
-    Returns token_prob [total_rows] (NaN on rows past n_sel_b L_b),
-    slot_accept [B, max_slots] int32 (0 past n_sel_b), accept_len [B] int32.
+    Returns token_prob [total_rows] (NaN outside every block),
+    slot_accept [B, max_slots] int32 (0 past n_slots[b]), accept_len [B] int32.
     ``rows`` restricts the per-row probabilities as in ``draft_select``."""
     x = np.asarray(logits)
-    nsel = np.asarray(n_selected, dtype=np.int64)
-    sl = np.asarray(slot_len, dtype=np.int64)
-    if row_offsets is None:
-        per = (np.asarray(n_slots, dtype=np.int64) if n_slots is not None else nsel) * sl
-        row_offsets = np.concatenate([[0], np.cumsum(per)])
-    offs = np.asarray(row_offsets, dtype=np.int64)
+    offs, ns, sl = _offsets(row_offsets, n_slots, slot_len)
     tok = np.asarray(tokens, dtype=np.int64)
-    B = nsel.size
+    B = ns.size
     total = int(x.shape[0])
     if max_slots is None:
-        max_slots = int(nsel.max()) if B else 0
+        max_slots = int(ns.max()) if B else 0
     active = np.zeros(total, dtype=bool)
     for b in range(B):
-        active[offs[b]: offs[b] + nsel[b] * sl[b]] = True
+        active[offs[b]: offs[b] + ns[b] * sl[b]] = True
     prob = np.full(total, np.nan)
     todo = range(total) if rows is None else [int(r) for r in rows]
     for g in todo:
@@ -291,7 +291,7 @@ def verify_accept(logits, tokens, n_selected, slot_len, *, temperature: float,
     slot_acc = np.zeros((B, max_slots), dtype=np.int32)
     acc = np.zeros(B, dtype=np.int32)
     for b in range(B):
-        n, L, o = int(nsel[b]), int(sl[b]), int(offs[b])
+        n, L, o = int(ns[b]), int(sl[b]), int(offs[b])
         sa, a = accept_prefix(prob[o: o + n * L], n, L, token_threshold)
         slot_acc[b, :n] = sa
         acc[b] = a

@@ -190,38 +190,50 @@ def test_draft_select_worked_example():
     # b0: only slot 0 above 0.8; b1: none above, most confident is slot 1
     assert out["slot_selected"].tolist() == [[1, 0, 0], [0, 1, 0]]
     assert out["n_selected"].tolist() == [1, 1]
-    assert out["verify_rows"].tolist() == [0, 1, -1, -1, -1, -1, 3, 4, 5, -1, -1, -1]
-    assert out["verify_tokens"].tolist() == [7, 8, -1, -1, -1, -1, 16, 17, 18, -1, -1, -1]
+    # verification block packed densely: b0's slot 0 (2 rows), b1's slot 1 (3 rows)
+    assert out["verify_row_offsets"].tolist() == [0, 2, 5]
+    assert out["verify_src_rows"].tolist() == [0, 1, 9, 10, 11] + [-1] * 7
+    assert out["verify_tokens"].tolist() == [7, 8, 16, 17, 18] + [-1] * 7
     # with a threshold of 0.5 b0 takes slots 0 and 2, b1 slot 1
     out = smp.draft_select(x, [3, 2], [2, 3], temperature=0.0, slot_threshold=0.5)
     assert out["slot_selected"].tolist() == [[1, 0, 1], [0, 1, 0]]
-    assert out["verify_rows"].tolist() == [0, 1, 4, 5, -1, -1, 3, 4, 5, -1, -1, -1]
-    assert out["verify_tokens"].tolist() == [7, 8, 11, 12, -1, -1, 16, 17, 18, -1, -1, -1]
+    assert out["verify_row_offsets"].tolist() == [0, 4, 7]
+    assert out["verify_src_rows"].tolist() == [0, 1, 4, 5, 9, 10, 11] + [-1] * 5
+    assert out["verify_tokens"].tolist() == [7, 8, 11, 12, 16, 17, 18] + [-1] * 5
 
 
 def test_verify_accept_worked_example():
-    # Verification of b0's 2 selected slots of 2 tokens (rows 0-3) and b1's
-    # 1 slot of 3 tokens (rows 6-8) in the draft layout (S_b L_b rows each).
+    # b0 verifies 2 slots of 2 tokens (rows 0-3), b1 one slot of 3 tokens
+    # (rows 4-6); two trailing rows belong to no block.
     V = 40
-    tokens = np.array([3, 9, 4, 1, -1, -1, 30, 31, 32, -1, -1, -1])
-    heights = {0: 2.0, 1: 5.0, 2: 6.0, 3: 1.0, 6: 4.0, 7: 4.5, 8: 0.0}
-    x = _peaked(V, [(r, int(tokens[r]), a) for r, a in heights.items()], 12)
-    out = smp.verify_accept(x, tokens, [2, 1], [2, 3], temperature=0.0, token_threshold=0.4,
-                            n_slots=[3, 2])
+    tokens = np.array([3, 9, 4, 1, 30, 31, 32, -1, -1])
+    heights = {0: 2.0, 1: 5.0, 2: 6.0, 3: 1.0, 4: 4.0, 5: 4.5, 6: 0.0}
+    x = _peaked(V, [(r, int(tokens[r]), a) for r, a in heights.items()], 9)
+    out = smp.verify_accept(x, tokens, [2, 1], [2, 3], temperature=0.0, token_threshold=0.4)
     p = {r: math.exp(a) / (math.exp(a) + V - 1) for r, a in heights.items()}
-    # p: row0 .159 (fails), row1 .792, row2 .912, row3 .065; row6 .583, row7 .698, row8 .025
+    # p: row0 .159 (fails), row1 .792, row2 .912, row3 .065; row4 .583, row5 .698, row6 .025
     for r in heights:
         assert abs(out["token_prob"][r] - p[r]) < 1e-14
-    assert np.isnan(out["token_prob"][[4, 5, 9, 10, 11]]).all()
+    assert np.isnan(out["token_prob"][[7, 8]]).all()
     assert out["slot_accept"].tolist() == [[0, 1], [2, 0]]
     assert out["accept_len"].tolist() == [0, 2]
+    # the same rows placed at explicit offsets with a gap between the sequences
+    xg = np.zeros((11, V))
+    xg[0:4], xg[6:9] = x[0:4], x[4:7]
+    tg = np.full(11, -1)
+    tg[0:4], tg[6:9] = tokens[0:4], tokens[4:7]
+    out2 = smp.verify_accept(xg, tg, [2, 1], [2, 3], temperature=0.0, token_threshold=0.4,
+                             row_offsets=[0, 6, 9])
+    assert out2["accept_len"].tolist() == [0, 2]
+    assert out2["slot_accept"].tolist() == [[0, 1], [2, 0]]
 
 
 def test_verify_of_own_draft_reproduces_draft_probability():
     rng = np.random.default_rng(3)
     x = rng.standard_normal((8, 300)) * 2
     d = smp.draft_select(x, [2], [4], temperature=0.8, slot_threshold=0.0, seed=4, offset=1)
-    v = smp.verify_accept(x, d["draft_tokens"], [2], [4], temperature=0.8, token_threshold=0.0)
+    assert d["verify_src_rows"].tolist() == list(range(8))
+    v = smp.verify_accept(x, d["verify_tokens"], [2], [4], temperature=0.8, token_threshold=0.0)
     assert np.allclose(v["token_prob"], d["draft_prob"], rtol=1e-13)
     assert v["accept_len"].tolist() == [8]
 
