@@ -79,6 +79,7 @@ typedef enum { ZARYA_BF16 = 0, ZARYA_FP32 = 1 } zarya_dtype;
 #define ZARYA_DEVERR_ACCEPT 4         /* accept_len[b] outside [0, R_b] */
 #define ZARYA_DEVERR_TIMEOUT 5        /* a pipeline wait gave up (no progress for ~2 s) */
 #define ZARYA_DEVERR_MASK_MODE 6      /* mask_mode[b] not a zarya_mask_mode */
+#define ZARYA_DEVERR_TOKEN 7          /* a verification token outside [0, vocab) */
 
 /* Shapes and host-known bounds shared by both calls. */
 typedef struct {
@@ -220,6 +221,105 @@ zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
                                        const int32_t* cache_lens, int32_t* new_lens,
                                        const int32_t* page_table, const zarya_attn_desc* desc,
                                        zarya_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Slot selection and token acceptance (Sec. 5.2 steps 3-6).
+ *
+ * The draft pass (step 3, ZARYA_MASK_BIDIR_BLOCK attention) yields logits for
+ * every block row. zarya_draft_select draws one token per row, takes each
+ * slot's confidence as the probability of the token drawn at its first row
+ * (step 3), and selects the slots to verify (step 5): those whose confidence
+ * exceeds slot_threshold, or, when none does, the single most confident one.
+ * It lays out the verification block: the selected slots' rows, in slot
+ * order, packed densely per sequence (n_selected[b] * L_b rows each), which is
+ * the q / k_new row layout of the verification attention pass.
+ *
+ * The verification pass (step 6, ZARYA_MASK_SLOT_CAUSAL or
+ * ZARYA_MASK_SLOT_INDEPENDENT attention over the verification block) yields
+ * logits for those rows. zarya_verify_accept takes the probability of each
+ * drafted token and accepts tokens while it exceeds token_threshold: per
+ * verified slot its accepted prefix, and over the whole verification block
+ * the accepted prefix length accept_len[b], which zarya_kv_append commits
+ * (step 7).
+ *
+ * Definitions used by both calls:
+ *  - Row probability of token t: softmax(x / T)[t] over the V logits x of the
+ *    row (softmax(x) when T = 0), computed in fp32.
+ *  - Draw (steps 3-4): T = 0: argmax of x. T > 0: Gumbel-max sampling, the
+ *    argmax of x / T + g_v with g_v standard Gumbel noise. Ties go to the
+ *    lowest vocabulary index; comparisons of probabilities with thresholds
+ *    are strict.
+ *  - Noise: g_v of logits row `row` comes from Philox4x32-10 (Salmon et al.,
+ *    SC'11) with key (seed low word, seed high word) and counter
+ *    (v / 4, row, offset low word, offset high word); word v % 4 of the
+ *    output is w, u = fl32(fl32(w) * 2^-32 + 2^-33) in (0, 1],
+ *    E = -log1p(-u), g_v = -log(E), in fp32.
+ *  - Logits rows: row r of the batch starts at element r * row_stride of
+ *    `logits` (bf16 or fp32, 16-byte aligned). Sequence b owns rows
+ *    row_offsets[b] .. row_offsets[b+1] - 1, which must number
+ *    n_slots[b] * slot_len[b] (device check: ZARYA_DEVERR_ROWS, and the
+ *    sequence is skipped); slot s of sequence b is its rows s*L_b .. s*L_b +
+ *    L_b - 1. Rows outside every sequence are not read.
+ */
+typedef struct {
+  int32_t batch;            /* B >= 1 */
+  int32_t vocab;            /* V >= 1 */
+  int32_t dtype;            /* zarya_dtype of the logits */
+  int32_t max_slots;        /* >= every S_b; row length of slot_conf, slot_selected, slot_accept */
+  int32_t total_rows;       /* rows of the logits buffer and of the per-row outputs;
+                               >= row_offsets[B] */
+  int32_t reserved;         /* must be 0 */
+  int64_t row_stride;       /* elements from one logits row to the next: >= vocab, and
+                               row_stride * element size a multiple of 16 bytes */
+  float temperature;        /* T >= 0 (finite); 0 draws the argmax */
+  float slot_threshold;     /* step 5 */
+  float token_threshold;    /* step 6 */
+  uint32_t reserved2;       /* must be 0 */
+  uint64_t seed;            /* Philox key */
+  uint64_t offset;          /* Philox counter words 2-3; a new value gives fresh noise */
+  const int32_t* row_offsets; /* device [B + 1], non-decreasing */
+} zarya_sample_desc;
+
+/*
+ * Steps 3-5. Inputs: logits [total_rows, row_stride]; n_slots, slot_len
+ * device [B] (S_b, L_b >= 1, S_b <= max_slots). Outputs (device, written):
+ *  draft_tokens       [total_rows] int32   drawn token of every block row
+ *  draft_prob         [total_rows] float   its probability
+ *  slot_conf          [B, max_slots] float confidence of slot s (0 for s >= S_b)
+ *  slot_selected      [B, max_slots] uint8 1 if slot s is selected
+ *  n_selected         [B] int32            selected slots (>= 1 for a valid sequence)
+ *  verify_row_offsets [B + 1] int32        verification layout: running sum of
+ *                                          n_selected[b] * L_b (starts at 0)
+ *  verify_src_rows    [total_rows] int32   verification row k -> the draft row it
+ *                                          verifies; -1 from verify_row_offsets[B] on
+ *  verify_tokens      [total_rows] int32   the token drafted at that row; -1 after
+ * Per-row outputs of rows outside every sequence are not written. A sequence
+ * that fails the device checks gets n_selected[b] = 0 (no verification rows).
+ */
+zarya_status zarya_draft_select(const void* logits, const int32_t* n_slots,
+                                const int32_t* slot_len, int32_t* draft_tokens,
+                                float* draft_prob, float* slot_conf, uint8_t* slot_selected,
+                                int32_t* n_selected, int32_t* verify_row_offsets,
+                                int32_t* verify_src_rows, int32_t* verify_tokens,
+                                const zarya_sample_desc* desc, zarya_stream_t stream);
+
+/*
+ * Step 6. desc->row_offsets is the verification layout (verify_row_offsets
+ * of the draft); n_slots[b] is the number of verified slots (n_selected of
+ * the draft, 0 allowed), slot_len[b] = L_b; tokens [total_rows] int32 holds
+ * the token of every verification row (verify_tokens of the draft).
+ * Outputs (device, written):
+ *  token_prob  [total_rows] float        probability of the row's token (0, with
+ *                                        ZARYA_DEVERR_TOKEN, for a token outside [0, V))
+ *  slot_accept [B, max_slots] int32      accepted prefix of verified slot k (0 past n_slots[b])
+ *  accept_len  [B] int32                 accepted prefix of the sequence's verification
+ *                                        rows (0 .. n_slots[b] * L_b)
+ * Rows outside every sequence are not read or written.
+ */
+zarya_status zarya_verify_accept(const void* logits, const int32_t* tokens,
+                                 const int32_t* n_slots, const int32_t* slot_len,
+                                 float* token_prob, int32_t* slot_accept, int32_t* accept_len,
+                                 const zarya_sample_desc* desc, zarya_stream_t stream);
 
 /*
  * Synchronises `stream`, then reads and clears the error word of the device

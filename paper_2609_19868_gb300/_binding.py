@@ -54,6 +54,26 @@ class AttnDesc(ctypes.Structure):
     ]
 
 
+class SampleDesc(ctypes.Structure):
+    """Mirror of ``zarya_sample_desc``."""
+    _fields_ = [
+        ("batch", ctypes.c_int32),
+        ("vocab", ctypes.c_int32),
+        ("dtype", ctypes.c_int32),
+        ("max_slots", ctypes.c_int32),
+        ("total_rows", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
+        ("row_stride", ctypes.c_int64),
+        ("temperature", ctypes.c_float),
+        ("slot_threshold", ctypes.c_float),
+        ("token_threshold", ctypes.c_float),
+        ("reserved2", ctypes.c_uint32),
+        ("seed", ctypes.c_uint64),
+        ("offset", ctypes.c_uint64),
+        ("row_offsets", ctypes.c_void_p),
+    ]
+
+
 _lib = None
 
 
@@ -80,6 +100,11 @@ def load() -> ctypes.CDLL:
     lib.zarya_kv_append.restype = ctypes.c_int
     lib.zarya_kv_append_commit_to.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, dp, vp]
     lib.zarya_kv_append_commit_to.restype = ctypes.c_int
+    sp = ctypes.POINTER(SampleDesc)
+    lib.zarya_draft_select.argtypes = [vp] * 11 + [sp, vp]
+    lib.zarya_draft_select.restype = ctypes.c_int
+    lib.zarya_verify_accept.argtypes = [vp] * 7 + [sp, vp]
+    lib.zarya_verify_accept.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
     lib.zarya_check_device_error.restype = ctypes.c_int
     lib.zarya_last_error.argtypes = []
@@ -256,6 +281,76 @@ def kv_append_commit_to(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, 
                                           _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_kv_append_commit_to")
+
+
+def make_sample_desc(*, batch: int, vocab: int, dtype: int, max_slots: int, total_rows: int,
+                     row_stride: int, temperature: float, slot_threshold: float,
+                     token_threshold: float, seed: int, offset: int,
+                     row_offsets: torch.Tensor) -> SampleDesc:
+    """Fill a ``zarya_sample_desc``; ``row_offsets`` (int32 [B + 1]) must stay alive."""
+    _check_cuda("row_offsets", row_offsets, torch.int32)
+    d = SampleDesc()
+    d.batch, d.vocab, d.dtype = int(batch), int(vocab), int(dtype)
+    d.max_slots, d.total_rows, d.reserved = int(max_slots), int(total_rows), 0
+    d.row_stride = int(row_stride)
+    d.temperature = float(temperature)
+    d.slot_threshold = float(slot_threshold)
+    d.token_threshold = float(token_threshold)
+    d.reserved2 = 0
+    d.seed = int(seed) & (2 ** 64 - 1)
+    d.offset = int(offset) & (2 ** 64 - 1)
+    d.row_offsets = row_offsets.data_ptr()
+    return d
+
+
+def _check_logits(logits, desc: SampleDesc):
+    if not isinstance(logits, torch.Tensor) or not logits.is_cuda:
+        raise TypeError("logits must be a CUDA tensor")
+    want = torch.bfloat16 if desc.dtype == BF16 else torch.float32
+    if logits.dtype != want:
+        raise TypeError(f"logits must be {want}, got {logits.dtype}")
+    if logits.dim() != 2 or logits.stride(1) != 1 or logits.stride(0) != desc.row_stride:
+        raise ValueError("logits must be [rows, V] with row stride desc.row_stride")
+    if logits.shape[0] < desc.total_rows or logits.shape[1] != desc.vocab:
+        raise ValueError("logits shape does not match the descriptor")
+
+
+def draft_select(logits, n_slots, slot_len, draft_tokens, draft_prob, slot_conf, slot_selected,
+                 n_selected, verify_row_offsets, verify_src_rows, verify_tokens,
+                 desc: SampleDesc, stream=None) -> None:
+    """``zarya_draft_select``: draws, slot confidences, slot selection and the
+    verification layout (Sec. 5.2 steps 3-5)."""
+    _check_logits(logits, desc)
+    for name, t in (("n_slots", n_slots), ("slot_len", slot_len), ("draft_tokens", draft_tokens),
+                    ("n_selected", n_selected), ("verify_row_offsets", verify_row_offsets),
+                    ("verify_src_rows", verify_src_rows), ("verify_tokens", verify_tokens)):
+        _check_cuda(name, t, torch.int32)
+    _check_cuda("draft_prob", draft_prob, torch.float32)
+    _check_cuda("slot_conf", slot_conf, torch.float32)
+    _check_cuda("slot_selected", slot_selected, torch.uint8)
+    st = load().zarya_draft_select(_ptr(logits), _ptr(n_slots), _ptr(slot_len), _ptr(draft_tokens),
+                                   _ptr(draft_prob), _ptr(slot_conf), _ptr(slot_selected),
+                                   _ptr(n_selected), _ptr(verify_row_offsets),
+                                   _ptr(verify_src_rows), _ptr(verify_tokens), ctypes.byref(desc),
+                                   _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_draft_select")
+
+
+def verify_accept(logits, tokens, n_slots, slot_len, token_prob, slot_accept, accept_len,
+                  desc: SampleDesc, stream=None) -> None:
+    """``zarya_verify_accept``: token probabilities and accepted prefixes of the
+    verification block (Sec. 5.2 step 6)."""
+    _check_logits(logits, desc)
+    for name, t in (("tokens", tokens), ("n_slots", n_slots), ("slot_len", slot_len),
+                    ("slot_accept", slot_accept), ("accept_len", accept_len)):
+        _check_cuda(name, t, torch.int32)
+    _check_cuda("token_prob", token_prob, torch.float32)
+    st = load().zarya_verify_accept(_ptr(logits), _ptr(tokens), _ptr(n_slots), _ptr(slot_len),
+                                    _ptr(token_prob), _ptr(slot_accept), _ptr(accept_len),
+                                    ctypes.byref(desc), _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_verify_accept")
 
 
 def check_device_error(stream=None) -> int:

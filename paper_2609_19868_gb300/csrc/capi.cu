@@ -14,7 +14,7 @@
 namespace zarya {
 namespace {
 
-constexpr int32_t kVersion = 100;  // 0.1.0
+constexpr int32_t kVersion = 200;  // 0.2.0
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
@@ -397,7 +397,66 @@ zarya_status kv_append_impl(const void* k_new, const void* v_new, const int32_t*
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the append kernel", ce);
 }
 
+zarya_status check_sample_desc(const zarya_sample_desc* d) {
+  if (d == nullptr) return ZARYA_ERR_INVALID_ARG;
+  if (d->batch < 1 || d->vocab < 1 || d->max_slots < 1 || d->total_rows < 1)
+    return ZARYA_ERR_INVALID_ARG;
+  if (d->dtype != ZARYA_BF16 && d->dtype != ZARYA_FP32) return ZARYA_ERR_INVALID_ARG;
+  if (d->reserved != 0 || d->reserved2 != 0) return ZARYA_ERR_INVALID_ARG;
+  const int eb = d->dtype == ZARYA_BF16 ? 2 : 4;
+  if (d->row_stride < d->vocab || (d->row_stride * eb) % 16 != 0) return ZARYA_ERR_INVALID_ARG;
+  if (!(d->temperature >= 0.f) || std::isinf(d->temperature)) return ZARYA_ERR_INVALID_ARG;
+  if (std::isnan(d->slot_threshold) || std::isnan(d->token_threshold))
+    return ZARYA_ERR_INVALID_ARG;
+  if (d->row_offsets == nullptr) return ZARYA_ERR_INVALID_ARG;
+  if (static_cast<long long>(d->batch) * d->max_slots > 0x7fffffffLL) return ZARYA_ERR_UNSUPPORTED;
+  return ZARYA_OK;
+}
+
 }  // namespace
+
+zarya_status zarya_draft_select(const void* logits, const int32_t* n_slots,
+                                const int32_t* slot_len, int32_t* draft_tokens,
+                                float* draft_prob, float* slot_conf, uint8_t* slot_selected,
+                                int32_t* n_selected, int32_t* verify_row_offsets,
+                                int32_t* verify_src_rows, int32_t* verify_tokens,
+                                const zarya_sample_desc* desc, zarya_stream_t stream_) {
+  zarya_status st = check_sample_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!logits || !n_slots || !slot_len || !draft_tokens || !draft_prob || !slot_conf ||
+      !slot_selected || !n_selected || !verify_row_offsets || !verify_src_rows || !verify_tokens)
+    return ZARYA_ERR_INVALID_ARG;
+  if (!aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, logits);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  const SampleCall c{logits, n_slots, slot_len, desc, sm_count()};
+  const DraftOutputs o{draft_tokens, draft_prob,         slot_conf,       slot_selected,
+                       n_selected,   verify_row_offsets, verify_src_rows, verify_tokens};
+  ce = launch_draft_select(c, o, err, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the draft-select kernels", ce);
+}
+
+zarya_status zarya_verify_accept(const void* logits, const int32_t* tokens,
+                                 const int32_t* n_slots, const int32_t* slot_len,
+                                 float* token_prob, int32_t* slot_accept, int32_t* accept_len,
+                                 const zarya_sample_desc* desc, zarya_stream_t stream_) {
+  zarya_status st = check_sample_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!logits || !tokens || !n_slots || !slot_len || !token_prob || !slot_accept || !accept_len)
+    return ZARYA_ERR_INVALID_ARG;
+  if (!aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, logits);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  const SampleCall c{logits, n_slots, slot_len, desc, sm_count()};
+  ce = launch_verify_accept(c, tokens, token_prob, slot_accept, accept_len, err, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the verify-accept kernels", ce);
+}
 
 zarya_status zarya_slot_attn(const void* q, const void* k_cache, const void* v_cache,
                              const int32_t* cache_lens, const int32_t* page_table,

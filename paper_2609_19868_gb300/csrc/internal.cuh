@@ -83,6 +83,32 @@ struct AppendParams {
   int rows_per_block;       // block rows copied by one CTA (gridDim.x CTAs per sequence)
 };
 
+// Common inputs of the slot-selection and token-acceptance calls.
+struct SampleCall {
+  const void* logits;
+  const int32_t* n_slots;
+  const int32_t* slot_len;
+  const zarya_sample_desc* desc;
+  int sms;  // multiprocessors of the device (sizes the row split)
+};
+
+struct DraftOutputs {
+  int32_t* draft_tokens;
+  float* draft_prob;
+  float* slot_conf;
+  uint8_t* slot_selected;
+  int32_t* n_selected;
+  int32_t* verify_row_offsets;
+  int32_t* verify_src_rows;
+  int32_t* verify_tokens;
+};
+
+cudaError_t launch_draft_select(const SampleCall& c, const DraftOutputs& o, int* err,
+                                cudaStream_t stream);
+cudaError_t launch_verify_accept(const SampleCall& c, const int32_t* tokens, float* token_prob,
+                                 int32_t* slot_accept, int32_t* accept_len, int* err,
+                                 cudaStream_t stream);
+
 // Dynamic shared memory of the tensor-core kernel.
 size_t tc_smem_bytes();
 

@@ -230,3 +230,124 @@ def make(name: str, small: bool = False, seed: Optional[int] = None, **override)
         q_row_offsets=i32(offs), page_table=page_table, q=q, k_cache=k_cache,
         v_cache=v_cache, k_new=k_new, v_new=v_new, scale=1.0 / math.sqrt(D),
         both_modes=both)
+
+
+# --------------------------------------------------------------------------
+# Logits for slot selection and token acceptance (Sec. 5.2 steps 3-6).
+#
+# Recipe (rng = numpy.random.default_rng(seed); integers and peak draws first,
+# in this order, then the base logits):
+#   1. slot lengths L_b (fixed or uniform choice from a set); S_b slots each
+#   2. verified slots n_b ~ uniform integer in [1, S_b] (the slot count of the
+#      verification block, whose rows are packed densely)
+#   3. per draft row: a peak with probability 0.7 at a uniform token, of
+#      height ~ U(10, 22)
+#   4. per verification row: its token, uniform in [0, V); a peak at that
+#      token with probability 0.8, of height ~ U(8, 20), else at a uniform token
+#   5. base logits ~ N(0, 2^2), drawn with torch.randn from a generator seeded
+#      with ``seed`` on the target device, in float32; peaks are added, then
+#      the values are rounded to the storage type (bf16 rounding makes ties
+#      of the row maximum common in rows without a peak).
+# With V = 151936 a row's softmax mass off the peak is about V e^2 ~ e^13.9,
+# so peak heights in [10, 22] give first-token confidences from ~0.02 to
+# ~1: both sides of the thresholds 0.9 / 0.4 occur.
+# The vocabulary size is that of the Qwen3 backbone Zarya builds on.
+
+QWEN3_VOCAB = 151936
+
+SAMPLE_SPECS = {
+    # small case for parity against the oracle: ragged V (not a multiple of 8)
+    "select_tiny": dict(seed=20, B=3, V=20011, dtype="fp32", n_slots=3,
+                        slot_len=("choice", (2, 3, 5))),
+    # the decode_small block (B8, 4 slots x 8 tokens) over the full vocabulary
+    "select_decode_small": dict(seed=21, B=8, V=QWEN3_VOCAB, dtype="bf16", n_slots=4,
+                                slot_len=("fixed", 8)),
+    # the serving_mix blocks (B64, 8 slots, L in {4, 8, 16, 32})
+    "select_serving_mix": dict(seed=22, B=64, V=QWEN3_VOCAB, dtype="bf16", n_slots=8,
+                               slot_len=("choice", (4, 8, 16, 32))),
+    # the long_ctx blocks (B4, 16 slots x 32 tokens)
+    "select_long_ctx": dict(seed=23, B=4, V=QWEN3_VOCAB, dtype="bf16", n_slots=16,
+                            slot_len=("fixed", 32)),
+}
+
+SLOT_THRESHOLD = 0.9    # Sec. 6 evaluation settings
+TOKEN_THRESHOLD = 0.4
+
+
+@dataclass
+class SamplingWorkload:
+    name: str
+    B: int
+    V: int
+    dtype: str
+    n_slots: np.ndarray         # int32 [B]   S_b of the draft block
+    slot_len: np.ndarray        # int32 [B]   L_b
+    row_offsets: np.ndarray     # int32 [B+1] draft layout (running sum of S_b L_b)
+    draft_logits: torch.Tensor  # [rows, V]
+    n_verify: np.ndarray        # int32 [B]   slots in the verification block
+    verify_offsets: np.ndarray  # int32 [B+1] running sum of n_b L_b
+    verify_tokens: np.ndarray   # int32 [verify rows]
+    verify_logits: torch.Tensor  # [verify rows, V]
+
+    @property
+    def rows(self) -> int:
+        return int(self.row_offsets[-1])
+
+    @property
+    def verify_rows(self) -> int:
+        return int(self.verify_offsets[-1])
+
+    @property
+    def max_slots(self) -> int:
+        return int(self.n_slots.max())
+
+
+def make_sampling(name: str, device="cpu", seed: Optional[int] = None,
+                  **override) -> SamplingWorkload:
+    """Build sampling workload ``name`` (SAMPLE_SPECS) with its logits on ``device``."""
+    spec = dict(SAMPLE_SPECS[name])
+    spec.update(override)
+    if seed is not None:
+        spec["seed"] = seed
+    rng = np.random.default_rng(spec["seed"])
+    B, V, S = spec["B"], spec["V"], spec["n_slots"]
+    kind = spec["slot_len"]
+    if kind[0] == "fixed":
+        L = np.full(B, kind[1], dtype=np.int64)
+    else:
+        L = rng.choice(np.asarray(kind[1], dtype=np.int64), size=B)
+    n_slots = np.full(B, S, dtype=np.int64)
+    n_ver = rng.integers(1, n_slots + 1)
+    offs = np.concatenate([[0], np.cumsum(n_slots * L)]).astype(np.int64)
+    voffs = np.concatenate([[0], np.cumsum(n_ver * L)]).astype(np.int64)
+    rows, vrows = int(offs[-1]), int(voffs[-1])
+    d_peak = rng.random(rows) < 0.7
+    d_tok = rng.integers(0, V, size=rows)
+    d_h = rng.uniform(10.0, 22.0, size=rows)
+    v_tok = rng.integers(0, V, size=vrows)
+    v_on = rng.random(vrows) < 0.8
+    v_other = rng.integers(0, V, size=vrows)
+    v_h = rng.uniform(8.0, 20.0, size=vrows)
+
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(spec["seed"]))
+    tdt = _torch_dtype(spec["dtype"])
+
+    def logits(n, peak_rows, peak_tok, peak_h):
+        x = torch.randn((n, V), generator=gen, device=device, dtype=torch.float32) * 2.0
+        if len(peak_rows):
+            r = torch.as_tensor(peak_rows, dtype=torch.int64, device=device)
+            t = torch.as_tensor(peak_tok, dtype=torch.int64, device=device)
+            h = torch.as_tensor(peak_h, dtype=torch.float32, device=device)
+            x[r, t] += h
+        return x.to(tdt)
+
+    pr = np.nonzero(d_peak)[0]
+    draft = logits(rows, pr, d_tok[pr], d_h[pr])
+    vt = np.where(v_on, v_tok, v_other)
+    verify = logits(vrows, np.arange(vrows), vt, v_h)
+    i32 = lambda a: np.ascontiguousarray(a, dtype=np.int32)  # noqa: E731
+    return SamplingWorkload(name=name, B=B, V=V, dtype=spec["dtype"], n_slots=i32(n_slots),
+                            slot_len=i32(L), row_offsets=i32(offs), draft_logits=draft,
+                            n_verify=i32(n_ver), verify_offsets=i32(voffs),
+                            verify_tokens=i32(v_tok), verify_logits=verify)

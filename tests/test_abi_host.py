@@ -167,3 +167,60 @@ def test_staged_rejects_missing_block_kv(lib):
                                     vp(None), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE), vp(None), 0,
                                     ctypes.byref(d), None)
     assert st == 1
+
+
+def _sdesc(**kw):
+    d = zb.SampleDesc()
+    base = dict(batch=2, vocab=1000, dtype=zb.BF16, max_slots=4, total_rows=16, reserved=0,
+                row_stride=1000, temperature=0.0, slot_threshold=0.9, token_threshold=0.4,
+                reserved2=0, seed=1, offset=0, row_offsets=0x100000)
+    base.update(kw)
+    for k, v in base.items():
+        setattr(d, k, v)
+    return d
+
+
+def test_sample_desc_layout_matches_c():
+    assert ctypes.sizeof(zb.SampleDesc) == 72
+    assert zb.SampleDesc.row_stride.offset == 24
+    assert zb.SampleDesc.seed.offset == 48
+    assert zb.SampleDesc.row_offsets.offset == 64
+
+
+def _draft(lib, d, logits=FAKE, out=FAKE):
+    vp = ctypes.c_void_p
+    return lib.zarya_draft_select(vp(logits), vp(FAKE), vp(FAKE), vp(out), vp(FAKE), vp(FAKE),
+                                  vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE),
+                                  None if d is None else ctypes.byref(d), None)
+
+
+def _verify(lib, d, logits=FAKE, tokens=FAKE):
+    vp = ctypes.c_void_p
+    return lib.zarya_verify_accept(vp(logits), vp(tokens), vp(FAKE), vp(FAKE), vp(FAKE), vp(FAKE),
+                                   vp(FAKE), None if d is None else ctypes.byref(d), None)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(batch=0), dict(vocab=0), dict(max_slots=0), dict(total_rows=0), dict(dtype=5),
+    dict(reserved=1), dict(reserved2=3),
+    dict(row_stride=999),                         # shorter than the vocabulary
+    dict(row_stride=1001),                        # bf16 rows not a multiple of 16 bytes
+    dict(dtype=zb.FP32, row_stride=1002),
+    dict(temperature=-0.5), dict(temperature=float("inf")), dict(temperature=float("nan")),
+    dict(slot_threshold=float("nan")), dict(token_threshold=float("nan")),
+    dict(row_offsets=0),
+])
+def test_sampling_rejects_invalid_descriptors(lib, bad):
+    assert _draft(lib, _sdesc(**bad)) == 1
+    assert _verify(lib, _sdesc(**bad)) == 1
+
+
+def test_sampling_rejects_null_and_misaligned_pointers(lib):
+    assert _draft(lib, None) == 1
+    assert _verify(lib, None) == 1
+    assert _draft(lib, _sdesc(), logits=None) == 1
+    assert _draft(lib, _sdesc(), out=None) == 1
+    assert _draft(lib, _sdesc(), logits=FAKE + 8) == 1
+    assert _verify(lib, _sdesc(), tokens=None) == 1
+    assert _verify(lib, _sdesc(), logits=FAKE + 4) == 1
+    assert _draft(lib, _sdesc(batch=65536, max_slots=65536)) == 2
