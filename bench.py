@@ -14,6 +14,10 @@ data touched between two uses of one copy exceeds the L2 cache.
 
 Prints one JSON line. `--impl reference` times the fp64 CPU oracle instead
 (rank 0 only), each step a bounded sample of the same workload.
+
+`--path select` measures slot selection and token acceptance (Sec. 5.2
+steps 3-6) instead: zarya_draft_select over a block's logits, then
+zarya_verify_accept over the verification block it laid out.
 """
 from __future__ import annotations
 
@@ -463,6 +467,254 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+SELECT_LABELS = {
+    "select_decode_small": "select_decode_small: B8, 4 slots x 8 tokens, V 151936 (Qwen3 vocabulary), "
+                           "bf16 logits, thresholds 0.9 / 0.4",
+    "select_serving_mix": "select_serving_mix: B64, 8 slots, slot_len in {4,8,16,32}, V 151936, "
+                          "bf16 logits, thresholds 0.9 / 0.4",
+    "select_long_ctx": "select_long_ctx: B4, 16 slots x 32 tokens, V 151936, bf16 logits, "
+                       "thresholds 0.9 / 0.4",
+}
+
+
+def run_select(args):
+    """Slot selection and token acceptance (Sec. 5.2 steps 3-6): one step =
+    zarya_draft_select over the draft block's logits, then zarya_verify_accept
+    over the verification block the draft laid out (its tokens and layout
+    taken from the draft's outputs on the device)."""
+    import torch
+    import torch.distributed as dist
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    if rank == 0:
+        zbuild.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2609_19868_gb300 import _binding as zb
+    from paper_2609_19868_gb300 import session
+    from paper_2609_19868_gb300 import workloads as wl
+
+    zb.load()
+    zb.check_device_error()
+    name = args.workload if args.workload in SELECT_LABELS else "select_decode_small"
+    seed = wl.SAMPLE_SPECS[name]["seed"] + 1000 * rank
+    w = wl.make_sampling(name, device=dev, seed=seed)
+    T = args.temperature
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    eb = 2 if w.dtype == "bf16" else 4
+    logit_bytes = (w.draft_logits.numel() + w.verify_logits.numel()) * eb
+    n_rot = max(1, math.ceil(3 * l2 / max(logit_bytes, 1))) if logit_bytes < 3 * l2 else 1
+    stream = torch.cuda.Stream(dev)
+    with torch.cuda.stream(stream):
+        rots = [session.upload_sampling(w, dev, temperature=T, seed=seed, offset=r, chain=True)
+                for r in range(n_rot)]
+    torch.cuda.synchronize()
+
+    def step(sb):
+        sb.draft(stream)
+        sb.verify(stream)
+
+    K, W = args.steps, args.warmup
+    with torch.cuda.stream(stream):
+        for i in range(max(W, n_rot)):
+            step(rots[i % n_rot])
+    torch.cuda.synchronize()
+    assert zb.check_device_error(stream) == 0
+    vrows = int(rots[0].verify_row_offsets[-1].item())
+    draft_bytes = w.rows * w.V * eb
+    verify_bytes = vrows * w.V * eb
+
+    def capture(fn, count):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for r in range(count):
+                fn(rots[r])
+        return g
+
+    full, tail = divmod(K, n_rot)
+    step_graph = capture(step, n_rot)
+    step_tail = capture(step, tail) if tail else None
+    draft_graph = capture(lambda sb: sb.draft(stream), n_rot)
+    draft_tail = capture(lambda sb: sb.draft(stream), tail) if tail else None
+
+    def run(graph, tail_graph):
+        for _ in range(full):
+            graph.replay()
+        if tail_graph is not None:
+            tail_graph.replay()
+
+    for _ in range(max(1, -(-W // n_rot))):
+        step_graph.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local).start() if args.clocks else None
+    if sampler:
+        time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        run(step_graph, step_tail)
+        end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    total_ms = max_over_ranks(start.elapsed_time(end), dev, world)
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        d0.record(stream)
+        run(draft_graph, draft_tail)
+        d1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop(t0, time.time()) if sampler else None
+    assert zb.check_device_error(stream) == 0
+    draft_ms = max_over_ranks(d0.elapsed_time(d1) / K, dev, world)
+
+    # End to end through the public API: every step copies its draft logits
+    # from pinned host memory, runs both calls, and reads accept_len and the
+    # drafted tokens back (the verification logits stay resident: they are the
+    # output of a forward pass that runs between the two calls on the device).
+    host = w.draft_logits.cpu().pin_memory()
+    out_tok = torch.empty(w.rows, dtype=torch.int32).pin_memory()
+    out_acc = torch.empty(w.B, dtype=torch.int32).pin_memory()
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in rots]
+    ev_done = [torch.cuda.Event() for _ in rots]
+
+    def e2e_steps(count):
+        s_in.wait_stream(stream)
+        s_out.wait_stream(stream)
+        for r in range(count):
+            sb = rots[r]
+            with torch.cuda.stream(s_in):
+                sb.draft_logits.copy_(host, non_blocking=True)
+                ev_in[r].record(s_in)
+            with torch.cuda.stream(stream):
+                stream.wait_event(ev_in[r])
+                step(sb)
+                ev_done[r].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_done[r])
+                out_tok.copy_(sb.draft_tokens, non_blocking=True)
+                out_acc.copy_(sb.accept_len, non_blocking=True)
+        stream.wait_stream(s_in)
+        stream.wait_stream(s_out)
+
+    with torch.cuda.stream(stream):
+        e2e_steps(n_rot)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        e2e_steps(n_rot)
+    gt = None
+    if tail:
+        gt = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gt, stream=stream):
+            e2e_steps(tail)
+    g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        run(g, gt)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev, world)
+    assert zb.check_device_error(stream) == 0
+
+    hbm_peak, _, peak_src = read_peaks()
+    draft_gbs = draft_bytes / (draft_ms * 1e-3) / 1e9
+    line = {
+        "metric": "slot select + token accept steps/s (draft select over the block's logits, "
+                  "then acceptance over the verification block)",
+        "value": round(replica_throughput(K, world, total_ms), 2),
+        "unit": "steps/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(total_ms / K, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32 (bf16 logits)",
+        "data": "synthetic (seeded N(0,2^2) logits with peaked tokens; no weights or datasets)",
+        "config": {
+            "workload": SELECT_LABELS[name],
+            "temperature": T,
+            "global_batch": w.B * world,
+            "draft_rows": w.rows,
+            "verify_rows": vrows,
+            "l2": (f"{n_rot} rotating logits copies of {logit_bytes / 1e6:.1f} MB (> L2 between "
+                   f"reuses)" if n_rot > 1 else
+                   f"logits {logit_bytes / 1e6:.0f} MB per step (> L2 {l2 / 1e6:.0f} MB)"),
+            "launch": f"CUDA graphs of {n_rot} steps (programmatic dependent launch)",
+        },
+        "roofline": {
+            "bound": "hbm" if T == 0 else "alu",
+            "achieved": round(draft_gbs, 1),
+            "peak": hbm_peak,
+            "unit": "GB/s",
+            "frac": round(draft_gbs / hbm_peak, 4),
+            "traffic": None,
+            "kernel": "zarya_draft_select (row pass + selection), per call",
+            "algorithmic_bytes": draft_bytes,
+            "peak_source": f"{peak_src} HBM copy bandwidth",
+        },
+        "e2e": {
+            "value": round(replica_throughput(K, world, e2e_ms), 2),
+            "unit": "steps/s",
+            "h2d_bytes_per_step": int(draft_bytes),
+            "d2h_bytes_per_step": int(4 * (w.rows + w.B)),
+        },
+        "gpu_launches": 4 * K,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = select_cpu_baseline(w, T, rots[0], budget_s=args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _oracle_select_rows(w, T, n_draft, n_verify, vtokens):
+    """The sampling oracle over the first n_draft draft rows and n_verify
+    verification rows (the per-row work dominates; the per-sequence rules are
+    negligible)."""
+    from oracle import sampling as smp
+
+    xd = w.draft_logits[:n_draft].float().cpu().numpy()
+    xv = w.verify_logits[:n_verify].float().cpu().numpy()
+    t0 = time.perf_counter()
+    smp.draft_select(xd, [n_draft], [1], temperature=T, slot_threshold=0.9, seed=1, fast=True,
+                     rows=range(n_draft))
+    smp.verify_accept(xv, vtokens[:n_verify], [n_verify], [1], temperature=T, token_threshold=0.4,
+                      rows=range(n_verify))
+    return time.perf_counter() - t0
+
+
+def select_cpu_baseline(w, T, sb, budget_s=20.0):
+    vrows = int(sb.verify_row_offsets[-1].item())
+    vt = sb.verify_tokens.cpu().numpy()
+    t1 = _oracle_select_rows(w, T, 1, 1, vt)
+    per_row = t1 / 2
+    n = int(max(1, min(w.rows, budget_s / 2 / max(per_row, 1e-6))))
+    nd, nv = n, min(n, max(vrows, 1))
+    t = _oracle_select_rows(w, T, nd, nv, vt)
+    frac_d, frac_v = nd / w.rows, nv / max(vrows, 1)
+    step_s = t / (nd + nv) * (w.rows + vrows)
+    return {"value": round(1.0 / step_s, 4), "unit": "steps/s", "cores": 1, "kind": "oracle",
+            "sample": f"{nd} of {w.rows} draft rows and {nv} of {vrows} verification rows "
+                      f"(numpy fp64 oracle), scaled to the whole step by rows"}
+
+
 def _oracle_step(oracle, w, seqs, threads=0):
     """The oracle's version of one step restricted to sequences ``seqs``."""
     from dataclasses import replace
@@ -565,20 +817,84 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_select_reference(args):
+    """The sampling oracle as the reference arm of --path select (rank 0)."""
+    world, rank, local = dist_setup()
+    if rank != 0:
+        return
+    from oracle import sampling as smp
+    from paper_2609_19868_gb300 import workloads as wl
+
+    name = args.workload if args.workload in SELECT_LABELS else "select_decode_small"
+    w = wl.make_sampling(name)
+    T = args.temperature
+    xv = w.verify_logits.float().numpy()
+    xd = w.draft_logits.float().numpy()
+    t0 = time.perf_counter()
+    smp.draft_select(xd[:1], [1], [1], temperature=T, slot_threshold=0.9, fast=True)
+    per_row = time.perf_counter() - t0
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    n = int(max(1, min(w.rows, budget / 2 / max(per_row, 1e-6))))
+    nv = min(n, w.verify_rows)
+
+    def one():
+        t = time.perf_counter()
+        smp.draft_select(xd[:n], [n], [1], temperature=T, slot_threshold=0.9, fast=True,
+                         rows=range(n))
+        smp.verify_accept(xv[:nv], w.verify_tokens[:nv], [nv], [1], temperature=T,
+                          token_threshold=0.4, rows=range(nv))
+        return time.perf_counter() - t
+
+    for _ in range(args.warmup):
+        one()
+    total = sum(one() for _ in range(args.steps))
+    step_s = total / args.steps / (n + nv) * (w.rows + w.verify_rows)
+    value = 1.0 / step_s
+    sample = (f"{n} of {w.rows} draft rows and {nv} of {w.verify_rows} verification rows per "
+              f"step (numpy fp64 oracle), scaled to the whole step by rows")
+    line = {
+        "impl": "reference",
+        "metric": "slot select + token accept steps/s (draft select over the block's logits, "
+                  "then acceptance over the verification block)",
+        "value": round(value, 4), "unit": "steps/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,2^2) logits with peaked tokens; no weights or datasets)",
+        "config": {"workload": SELECT_LABELS[name], "temperature": T, "global_batch": w.B},
+        "cpu_baseline": {"value": round(value, 4), "unit": "steps/s", "cores": 1,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="decode_small", choices=list(WORKLOAD_LABELS))
+    ap.add_argument("--workload", default=None,
+                    choices=list(WORKLOAD_LABELS) + list(SELECT_LABELS))
+    ap.add_argument("--path", choices=["attention", "select"], default="attention",
+                    help="attention: the slot-decode layer step (stage + attention + commit); "
+                         "select: slot selection + token acceptance over logits")
+    ap.add_argument("--temperature", type=float, default=0.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-clocks", dest="clocks", action="store_false")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    if args.impl == "reference":
+    if args.workload is None:
+        args.workload = "select_decode_small" if args.path == "select" else "decode_small"
+    if args.path == "select":
+        if args.impl == "reference":
+            run_select_reference(args)
+        else:
+            run_select(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

@@ -18,9 +18,11 @@
 // running sum over the batch) selects the slots (step 5) and lays out the
 // verification block; the verification form (one warp per sequence) scans the
 // accepted prefixes (step 6).
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <cstddef>
+#include <cstring>
 #include <cstdint>
 
 #include "internal.cuh"
@@ -80,6 +82,12 @@ __device__ __forceinline__ float ex2(float x) {
 }
 
 __device__ __forceinline__ float bf16_bits_to_f32(uint32_t b) { return __uint_as_float(b << 16); }
+
+__device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
+  __nv_bfloat162 r;
+  memcpy(&r, &w, sizeof r);
+  return r;
+}
 
 // Philox4x32 with 10 rounds (Salmon et al., SC'11): each round multiplies
 // counter words 0 and 2 by the round constants into 64-bit products and
@@ -181,18 +189,7 @@ __device__ __forceinline__ void absorb(RowState& st, const float (&x)[kN], int v
 // and one rescale test per chunk, and independent partial sums.
 template <int kMode, int kN>
 __device__ __forceinline__ void absorb_chunk(RowState& st, const float (&x)[kVecsPerThread][kN],
-                                             int e0, int estride, float k2) {
-  float vk[kVecsPerThread];
-#pragma unroll
-  for (int k = 0; k < kVecsPerThread; ++k) {
-    float m0 = fmaxf(x[k][0], x[k][1]);
-#pragma unroll
-    for (int j = 2; j < kN; j += 2) m0 = fmaxf(m0, fmaxf(x[k][j], x[k][j + 1]));
-    vk[k] = m0;
-  }
-  float vm = vk[0];
-#pragma unroll
-  for (int k = 1; k < kVecsPerThread; ++k) vm = fmaxf(vm, vk[k]);
+                                             float vm, int e0, int estride, float k2) {
   if (vm > st.m) {
     if (kMode == kDraftArgmax) {
       int best = 0x7fffffff;
@@ -299,6 +296,31 @@ __device__ __forceinline__ void widen(const uint4& v, float (&x)[16 / sizeof(TIn
     x[1] = __uint_as_float(v.y);
     x[2] = __uint_as_float(v.z);
     x[3] = __uint_as_float(v.w);
+  }
+}
+
+// Maximum of a thread's vectors of one stage: bf16 pairs compared packed
+// (the maximum of bf16 values is exact in either form), fp32 elementwise.
+template <typename TIn>
+__device__ __forceinline__ float chunk_max(const uint4 (&v)[kVecsPerThread],
+                                           const float (&x)[kVecsPerThread][16 / sizeof(TIn)]) {
+  if (sizeof(TIn) == 2) {
+    __nv_bfloat162 m2 = as_bf162(v[0].x);
+#pragma unroll
+    for (int k = 0; k < kVecsPerThread; ++k) {
+      if (k > 0) m2 = __hmax2(m2, as_bf162(v[k].x));
+      m2 = __hmax2(m2, as_bf162(v[k].y));
+      m2 = __hmax2(m2, as_bf162(v[k].z));
+      m2 = __hmax2(m2, as_bf162(v[k].w));
+    }
+    return fmaxf(__low2float(m2), __high2float(m2));
+  } else {
+    float m = x[0][0];
+#pragma unroll
+    for (int k = 0; k < kVecsPerThread; ++k)
+#pragma unroll
+      for (int j = 0; j < 16 / static_cast<int>(sizeof(TIn)); ++j) m = fmaxf(m, x[k][j]);
+    return m;
   }
 }
 
@@ -425,7 +447,7 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) row_pass_kernel(co
         float x[kVecsPerThread][kEpv];
 #pragma unroll
         for (int k = 0; k < kVecsPerThread; ++k) widen<TIn>(v[k], x[k]);
-        absorb_chunk<kMode>(st, x, e0, kConsumers * kEpv, a.k2);
+        absorb_chunk<kMode>(st, x, chunk_max<TIn>(v, x), e0, kConsumers * kEpv, a.k2);
       }
     }
     // Ragged tail: V % kEpv elements, on the last rank.
