@@ -1,11 +1,12 @@
 """Slot-decode step benchmark (one layer of Zarya Mode B, Sec. 5.2).
 
 One step = the whole hot path over one batch:
-  stage   zarya_kv_append(STAGE)   the block's K/V -> cache positions P_b..
-  attend  zarya_slot_attn          block rows over prefix + block (mask per sequence)
-  commit  zarya_kv_append(COMMIT)  accepted rows -> cache, P_b += accepted
-then the committed lengths are restored (a 4*B-byte device copy) so every
-step sees the same prefix lengths.
+  stage + attend  zarya_slot_attn_staged  the block's K/V -> cache positions
+                  P_b.., then block rows over prefix + block (mask per sequence)
+  commit          zarya_kv_commit_staged  P_b += accepted (the accepted rows,
+                  first in the block, are already in place)
+The commit writes the advanced lengths into a second array (a decoding
+loop's ping-pong), so every step sees the same prefix lengths.
 
 Default workload: decode_small (B8, 16/8 heads, D128, bf16, P=2048,
 contiguous cache, 4 slots x 8 tokens, slot-causal). Inputs are seeded and
@@ -256,9 +257,10 @@ def run_ours(args):
     torch.cuda.synchronize()
 
     def step(db):
-        # stage the block's own K/V and attend in one launch, then commit
+        # stage the block's own K/V and attend in one launch; the accepted
+        # rows are then already in place, so the commit advances the lengths
         db.stage_and_attend(stream)
-        db.commit(stream, new_lens=lens_next[id(db)])
+        db.commit_staged(stream, new_lens=lens_next[id(db)])
 
     K, W = args.steps, args.warmup
     with torch.cuda.stream(stream):
@@ -456,7 +458,7 @@ def run_ours(args):
             "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h),
         },
-        "gpu_launches": 2 * K,   # staged attention, commit copy (with the length advance)
+        "gpu_launches": 2 * K,   # staged attention, commit (length advance)
         "clocks": clocks,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -222,6 +222,24 @@ zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
                                        const int32_t* page_table, const zarya_attn_desc* desc,
                                        zarya_stream_t stream);
 
+/*
+ * Step 7 for a block whose rows are already in the cache: after the
+ * verification pass staged its block (zarya_slot_attn_staged, or
+ * zarya_kv_append with ZARYA_APPEND_STAGE, from the same k_new / v_new whose
+ * accepted rows come first), rows 0 .. accept_len[b] - 1 of the block already
+ * sit at positions P_b .. P_b + accept_len[b] - 1, so the commit only
+ * advances the length: new_lens[b] = cache_lens[b] + accept_len[b]. No cache
+ * byte moves; afterwards the cache holds exactly what zarya_kv_append_commit_to
+ * would leave in positions below new_lens[b]. accept_len, cache_lens: device
+ * [B] (read); new_lens: device [B] (written; may be cache_lens). The device
+ * checks and error behaviour are those of zarya_kv_append (a sequence that
+ * fails keeps its new_lens entry and sets the error word). Waits for the
+ * work queued before it on `stream`.
+ */
+zarya_status zarya_kv_commit_staged(const int32_t* accept_len, const int32_t* cache_lens,
+                                    int32_t* new_lens, const zarya_attn_desc* desc,
+                                    zarya_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Slot selection and token acceptance (Sec. 5.2 steps 3-6).
  *

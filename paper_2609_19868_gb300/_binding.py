@@ -100,6 +100,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_kv_append.restype = ctypes.c_int
     lib.zarya_kv_append_commit_to.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, dp, vp]
     lib.zarya_kv_append_commit_to.restype = ctypes.c_int
+    lib.zarya_kv_commit_staged.argtypes = [vp, vp, vp, dp, vp]
+    lib.zarya_kv_commit_staged.restype = ctypes.c_int
     sp = ctypes.POINTER(SampleDesc)
     lib.zarya_draft_select.argtypes = [vp] * 11 + [sp, vp]
     lib.zarya_draft_select.restype = ctypes.c_int
@@ -281,6 +283,18 @@ def kv_append_commit_to(k_new, v_new, accept_len, k_cache, v_cache, cache_lens, 
                                           _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_kv_append_commit_to")
+
+
+def kv_commit_staged(accept_len, cache_lens, new_lens, desc: AttnDesc, stream=None) -> None:
+    """``zarya_kv_commit_staged``: the commit of a block already staged in the
+    cache, new_lens = cache_lens + accept_len (Sec. 5.2 step 7)."""
+    _check_cuda("accept_len", accept_len, torch.int32)
+    _check_cuda("cache_lens", cache_lens, torch.int32)
+    _check_cuda("new_lens", new_lens, torch.int32)
+    st = load().zarya_kv_commit_staged(_ptr(accept_len), _ptr(cache_lens), _ptr(new_lens),
+                                       ctypes.byref(desc), _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_kv_commit_staged")
 
 
 def make_sample_desc(*, batch: int, vocab: int, dtype: int, max_slots: int, total_rows: int,

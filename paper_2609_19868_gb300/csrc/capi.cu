@@ -500,6 +500,31 @@ zarya_status zarya_kv_append_commit_to(const void* k_new, const void* v_new,
                         page_table, true, desc, stream);
 }
 
+zarya_status zarya_kv_commit_staged(const int32_t* accept_len, const int32_t* cache_lens,
+                                    int32_t* new_lens, const zarya_attn_desc* desc,
+                                    zarya_stream_t stream_) {
+  zarya_status st = check_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!accept_len || !cache_lens || !new_lens) return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, cache_lens);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  AppendParams p{};
+  p.accept_len = accept_len;
+  p.cache_lens = cache_lens;
+  p.new_lens = new_lens;
+  p.q_row_offsets = desc->q_row_offsets;
+  p.err = err;
+  p.B = desc->batch;
+  p.max_rows = desc->max_rows;
+  p.total_rows = desc->total_rows;
+  p.capacity = desc->cache_capacity;
+  ce = launch_commit_lens(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the commit kernel", ce);
+}
+
 zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {
   if (code) *code = 0;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);

@@ -117,6 +117,9 @@ cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map
                                 cudaStream_t stream);
 cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream);
 cudaError_t launch_kv_append(const AppendParams& p, bool commit, cudaStream_t stream);
+// new_lens[b] = cache_lens[b] + accept_len[b] after the device checks of the
+// append (the block's rows are already in the cache).
+cudaError_t launch_commit_lens(const AppendParams& p, cudaStream_t stream);
 
 // Bytes at the end of the attention workspace that hold the split counters
 // (which must be zero before a call); 0 when the plan needs no workspace.

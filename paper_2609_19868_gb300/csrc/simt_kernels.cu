@@ -143,6 +143,7 @@ slot_attn_f32_kernel(const SimtParams p) {
 // advance cache_lens[b] inside one thread-block cluster.
 constexpr int kAppendMaxCtasPerSeq = 8;
 constexpr int kAppendThreads = 256;
+constexpr int kCommitThreads = 128;
 constexpr int kAppendUnroll = 4;   // 16-byte vectors of K and of V in flight per thread
 
 // Copies rows i < accept_len[b] of the block (rows [x * rows_per_block, ...)
@@ -221,7 +222,35 @@ kv_append_copy_kernel(const AppendParams p) {
   }
 }
 
+// Commit of a block whose rows the verification pass already staged at
+// positions P_b.. (Sec. 5.2 step 7 with nothing left to copy): one thread per
+// sequence checks accept_len[b] and writes new_lens[b] = P_b + accept_len[b].
+// It waits for the kernel before it (accept_len comes from the acceptance
+// step, and new_lens may be the cache_lens that kernel reads).
+__global__ void __launch_bounds__(kCommitThreads) commit_lens_kernel(const AppendParams p) {
+  grid_dependency_wait();
+  grid_launch_dependents();
+  const int b = blockIdx.x * kCommitThreads + threadIdx.x;
+  if (b >= p.B) return;
+  const int P = p.cache_lens[b];
+  const int row0 = p.q_row_offsets[b];
+  const int R = p.q_row_offsets[b + 1] - row0;
+  const int a = p.accept_len[b];
+  int code = 0;
+  if (R < 0 || R > p.max_rows || row0 < 0 || row0 + R > p.total_rows) code = ZARYA_DEVERR_ROWS;
+  else if (a < 0 || a > R) code = ZARYA_DEVERR_ACCEPT;
+  else if (P < 0 || static_cast<long long>(P) + a > p.capacity) code = ZARYA_DEVERR_CAPACITY;
+  if (code != 0) record_error(p.err, code);
+  else p.new_lens[b] = P + a;
+}
+
 }  // namespace
+
+cudaError_t launch_commit_lens(const AppendParams& p, cudaStream_t stream) {
+  PdlLaunch l(dim3(static_cast<unsigned>((p.B + kCommitThreads - 1) / kCommitThreads)),
+              dim3(kCommitThreads), 0, stream);
+  return cudaLaunchKernelEx(&l.cfg, commit_lens_kernel, p);
+}
 
 cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream) {
   const long long warps = static_cast<long long>(p.B) * p.Hq * p.max_rows;

@@ -10,6 +10,8 @@ a step, all of which run in the library's kernels:
   stage()   zarya_kv_append(STAGE): block K/V -> cache positions P_b..
   attend()  zarya_slot_attn: out <- attention of the block over prefix+block
   commit()  zarya_kv_append(COMMIT): accepted rows -> cache, P_b += accepted
+  commit_staged()  zarya_kv_commit_staged: P_b += accepted, for a block
+            already staged (its accepted rows are in place)
 """
 from __future__ import annotations
 
@@ -66,6 +68,14 @@ class DeviceBatch:
             zb.kv_append_commit_to(self.k_new, self.v_new, self.accept_len, self.k_cache,
                                    self.v_cache, self.cache_lens, new_lens, self.page_table,
                                    self.desc, stream=stream)
+
+    def commit_staged(self, stream=None, new_lens=None) -> None:
+        """The commit after ``stage_and_attend`` (or ``stage``) of this block:
+        its accepted rows are already in the cache, so only the lengths
+        advance (in place, or into ``new_lens``)."""
+        zb.kv_commit_staged(self.accept_len, self.cache_lens,
+                            self.cache_lens if new_lens is None else new_lens, self.desc,
+                            stream=stream)
 
 
 def _i32(a, device) -> torch.Tensor:

@@ -156,6 +156,17 @@ def test_commit_to_rejects_invalid_calls(lib):
     assert app(k_cache=FAKE + 8) == 1
 
 
+def test_commit_staged_rejects_invalid_calls(lib):
+    vp = ctypes.c_void_p
+    d = _desc()
+    assert lib.zarya_kv_commit_staged(vp(None), vp(FAKE), vp(FAKE), ctypes.byref(d), None) == 1
+    assert lib.zarya_kv_commit_staged(vp(FAKE), vp(None), vp(FAKE), ctypes.byref(d), None) == 1
+    assert lib.zarya_kv_commit_staged(vp(FAKE), vp(FAKE), vp(None), ctypes.byref(d), None) == 1
+    assert lib.zarya_kv_commit_staged(vp(FAKE), vp(FAKE), vp(FAKE), None, None) == 1
+    assert lib.zarya_kv_commit_staged(vp(FAKE), vp(FAKE), vp(FAKE),
+                                      ctypes.byref(_desc(batch=0)), None) == 1
+
+
 def test_staged_rejects_missing_block_kv(lib):
     vp = ctypes.c_void_p
     d = _desc()

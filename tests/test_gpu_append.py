@@ -86,6 +86,51 @@ def test_commit_to_second_array_leaves_lengths_alone(zs, oracle_mod, name, small
     assert np.array_equal(new_lens.cpu().numpy(), lens2)
 
 
+@pytest.mark.parametrize("name,small", [(n, True) for n in wl.ORDER] +
+                         [("long_ctx", False), ("serving_mix", False)])
+def test_commit_staged_equals_copy_commit(zs, oracle_mod, name, small):
+    """zarya_kv_commit_staged after staging leaves the cache the copy commit
+    leaves (the accepted rows are already in place) and the same lengths."""
+    session, zb = zs
+    w = wl.make(name, small=small)
+    db = session.upload(w, "cuda")
+    db.stage()
+    new_lens = torch.full_like(db.cache_lens, -7)
+    db.commit_staged(new_lens=new_lens)
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    kc, vc, kc2, vc2, lens2 = _oracle_stage_commit(oracle_mod, w)
+    # the oracle's copy commit after staging rewrites rows that are already there
+    assert np.array_equal(kc.view(np.uint8), kc2.view(np.uint8))
+    gk, gv = _bits(db.k_cache), _bits(db.v_cache)
+    assert np.array_equal(gk, kc2.view(gk.dtype))
+    assert np.array_equal(gv, vc2.view(gv.dtype))
+    assert np.array_equal(new_lens.cpu().numpy(), lens2)
+    assert np.array_equal(db.cache_lens.cpu().numpy(), w.cache_lens)
+    # in place
+    db.commit_staged()
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    assert np.array_equal(db.cache_lens.cpu().numpy(), lens2)
+
+
+def test_commit_staged_checks(zs):
+    session, zb = zs
+    w = wl.make("decode_small", small=True)
+    db = session.upload(w, "cuda")
+    new_lens = torch.full_like(db.cache_lens, -7)
+    db.accept_len[1] = int(w.R[1]) + 1
+    db.commit_staged(new_lens=new_lens)
+    assert zb.check_device_error() == 4          # ZARYA_DEVERR_ACCEPT
+    got = new_lens.cpu().numpy()
+    assert got[1] == -7
+    assert all(got[b] == w.cache_lens[b] + w.accept_len[b] for b in range(w.B) if b != 1)
+    db = session.upload(w, "cuda")
+    db.cache_lens[0] = w.capacity - 2
+    db.commit_staged()
+    assert zb.check_device_error() == 3          # ZARYA_DEVERR_CAPACITY
+
+
 def test_commit_to_skips_a_failing_sequence(zs):
     session, zb = zs
     w = wl.make("decode_small", small=True)
