@@ -346,6 +346,38 @@ __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* 
   return true;
 }
 
+// L2 prefetch of the first kStagesK tiles of this CTA's key range (and of its
+// Q tile when map_q is given), from a reading of the sequence's lengths that
+// may be stale; nothing is prefetched when that reading is out of range.
+__device__ __forceinline__ void prefetch_first_tiles(const CUtensorMap* map_kv,
+                                                     const CUtensorMap* map_q, const TcParams& p,
+                                                     int b, int kvh, int mt, int split) {
+  const int P = ld_relaxed_gpu(p.cache_lens + b);
+  const long long R64 = static_cast<long long>(ld_relaxed_gpu(p.n_slots + b)) *
+                        ld_relaxed_gpu(p.slot_len + b);
+  const int mode = ld_relaxed_gpu(p.mask_mode + b);
+  const int row0 = ld_relaxed_gpu(p.q_row_offsets + b);
+  if (P < 0 || R64 < 1 || R64 > p.max_rows || P + R64 > p.capacity) return;
+  const int R = static_cast<int>(R64);
+  const int rows_per_tile = kBlockM / p.g;
+  const int r0 = mt * rows_per_tile;
+  if (r0 >= R) return;
+  const int r_hi = min(r0 + rows_per_tile, R) - 1;
+  const int kv_end = mode == ZARYA_MASK_BIDIR_BLOCK ? P + R : P + r_hi + 1;
+  const int n_tiles = (kv_end + kBlockN - 1) / kBlockN;
+  const int per_split = max(1, (n_tiles + p.splits - 1) / p.splits);
+  const int t_begin = split * per_split;
+  const int t_end = min(n_tiles, t_begin + min(per_split, kStagesK));
+  for (int t = t_begin; t < t_end; ++t) {
+    tma_prefetch_l2_4d(map_kv, 0, kvh, t * kBlockN, b);
+    tma_prefetch_l2_4d(map_kv, 64, kvh, t * kBlockN, b);
+  }
+  if (map_q != nullptr && row0 >= 0 && row0 + r0 < p.total_rows) {
+    tma_prefetch_l2_3d(map_q, 0, kvh * p.g, row0 + r0);
+    tma_prefetch_l2_3d(map_q, 64, kvh * p.g, row0 + r0);
+  }
+}
+
 // After a failed produce_range: let this CTA's own copies land before the CTA
 // (and its shared memory) goes away.
 __device__ __forceinline__ void drain_ring(uint64_t* full, int stages, int issued, int lane) {
@@ -412,6 +444,14 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     named_bar_sync(kBarProducers, 64);
     named_bar_arrive(kBarSetup, kThreads);
   }
+  // Before waiting for the kernel launched before this one, warm L2 with Q
+  // and the first tiles of this split's K / V. L2 is the point of coherence,
+  // so a prefetch cannot hand stale data to the loads made after the wait;
+  // the lengths read here (that kernel may still be writing them) only steer
+  // which lines are warmed. Contiguous caches only.
+  if ((warp == 0 || warp == 2) && lane == 0 && p.page_size == 0)
+    prefetch_first_tiles(warp == 0 ? &map_k : &map_v, warp == 0 ? &map_q : nullptr, p, b, kvh,
+                         mt, split);
   // Inputs may be written by the kernel launched before this one.
   grid_dependency_wait();
 
