@@ -51,6 +51,7 @@ namespace zarya {
 namespace {
 
 constexpr int kThreads = 384;
+constexpr int kSoftmaxWarps = 8;   // warps 4..11: two softmax warpgroups
 constexpr int kStagesK = 3;
 constexpr int kStagesV = 3;
 constexpr uint32_t kHalfBytes = kBlockN * 64 * 2;   // 128 rows x 128 B
@@ -76,6 +77,7 @@ struct Bars {
   uint64_t drain;
   uint64_t kfree;   // this CTA's last Q*K^T has completed: its K ring is idle
   uint64_t staged;  // staged attention: the block rows this CTA reads are in the cache
+  uint64_t stage_issued;  // staged attention: the first round of staging loads is issued
   uint64_t ready;   // cluster merge: every partial row this CTA owns has landed
   uint64_t go;      // cluster merge: every other split's K ring is free to receive
   uint32_t tmem_base;
@@ -239,55 +241,74 @@ __device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity,
 // vectors of each tensor per lane in flight per round, then fences the writes
 // against the async proxy; the producers wait on `staged` before loading the
 // first tile that holds one of these rows.
-struct WarpStager {
+// Staged attention: the block rows this CTA reads are copied from k_new /
+// v_new into the cache by the eight softmax warps (idle until the first score
+// tile). The loads of the first round are issued before the producers' first
+// tensor copies (16-byte loads issued behind this SM's tensor streams return
+// only when those streams end); the stores, any further rounds and the proxy
+// fence follow the set-up barrier.
+struct GroupStager {
   static constexpr int kVec = kHeadDim * 2 / 16;   // 16-byte vectors per (token, head) row
-  static constexpr int kRound = 12;
+  static constexpr int kThreads = kSoftmaxWarps * 32;
+  static constexpr int kRound = 2;                 // vectors of K and of V per thread per round
+  uint4 vk[kRound], vv[kRound];
+  long long d[kRound];
 
-  __device__ __forceinline__ static void run(const TcParams& p, int b, int kvh, int row0, int P,
-                                             int i_lo, int i_hi, int lane) {
+  __device__ __forceinline__ void load(const TcParams& p, int b, int kvh, int row0, int P,
+                                       int i_lo, int i_hi, int t, int base) {
     const uint4* kn = static_cast<const uint4*>(p.k_new);
     const uint4* vn = static_cast<const uint4*>(p.v_new);
-    uint4* kc = static_cast<uint4*>(p.k_cache);
-    uint4* vc = static_cast<uint4*>(p.v_cache);
     const int n = (i_hi - i_lo) * kVec;
-    for (int base = 0; base < n; base += kRound * 32) {
-      uint4 vk[kRound], vv[kRound];
-      long long d[kRound];
 #pragma unroll
-      for (int u = 0; u < kRound; ++u) {
-        const int idx = base + u * 32 + lane;
-        d[u] = -1;
-        if (idx < n) {
-          const int i = i_lo + idx / kVec;
-          const int c = idx % kVec;
-          const int t = P + i;
-          long long tr = -1;
-          if (p.page_size == 0) {
-            tr = static_cast<long long>(b) * p.capacity + t;
-          } else {
-            const int page =
-                p.page_table[static_cast<long long>(b) * p.max_pages + t / p.page_size];
-            if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
-            else tr = static_cast<long long>(page) * p.page_size + t % p.page_size;
-          }
-          if (tr >= 0) {
-            const long long sidx = (static_cast<long long>(row0 + i) * p.Hkv + kvh) * kVec + c;
-            vk[u] = __ldg(kn + sidx);
-            vv[u] = __ldg(vn + sidx);
-            d[u] = (tr * p.Hkv + kvh) * kVec + c;
-          }
+    for (int u = 0; u < kRound; ++u) {
+      const int idx = base + u * kThreads + t;
+      d[u] = -1;
+      if (idx < n) {
+        const int i = i_lo + idx / kVec;
+        const int c = idx % kVec;
+        const int tok = P + i;
+        long long tr = -1;
+        if (p.page_size == 0) {
+          tr = static_cast<long long>(b) * p.capacity + tok;
+        } else {
+          const int page =
+              p.page_table[static_cast<long long>(b) * p.max_pages + tok / p.page_size];
+          if (page < 0 || page >= p.n_pages) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+          else tr = static_cast<long long>(page) * p.page_size + tok % p.page_size;
         }
-      }
-#pragma unroll
-      for (int u = 0; u < kRound; ++u) {
-        if (d[u] >= 0) {
-          kc[d[u]] = vk[u];
-          vc[d[u]] = vv[u];
+        if (tr >= 0) {
+          const long long sidx = (static_cast<long long>(row0 + i) * p.Hkv + kvh) * kVec + c;
+          vk[u] = __ldg(kn + sidx);
+          vv[u] = __ldg(vn + sidx);
+          d[u] = (tr * p.Hkv + kvh) * kVec + c;
         }
       }
     }
+  }
+
+  __device__ __forceinline__ void store(const TcParams& p) {
+    uint4* kc = static_cast<uint4*>(p.k_cache);
+    uint4* vc = static_cast<uint4*>(p.v_cache);
+#pragma unroll
+    for (int u = 0; u < kRound; ++u) {
+      if (d[u] >= 0) {
+        kc[d[u]] = vk[u];
+        vc[d[u]] = vv[u];
+      }
+    }
+  }
+
+  // Stores the first round, copies the rest, and makes the writes visible to
+  // the tensor copies that will read them.
+  __device__ __forceinline__ void finish(const TcParams& p, int b, int kvh, int row0, int P,
+                                         int i_lo, int i_hi, int t) {
+    store(p);
+    const int n = (i_hi - i_lo) * kVec;
+    for (int base = kRound * kThreads; base < n; base += kRound * kThreads) {
+      load(p, b, kvh, row0, P, i_lo, i_hi, t, base);
+      store(p);
+    }
     asm volatile("fence.proxy.async.global;" ::: "memory");
-    __syncwarp();
   }
 };
 
@@ -431,7 +452,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     mbar_init(&bars->o_done[1], 1);
     mbar_init(&bars->drain, 1);
     mbar_init(&bars->kfree, 1);
-    mbar_init(&bars->staged, 1);
+    mbar_init(&bars->staged, kSoftmaxWarps);
+    mbar_init(&bars->stage_issued, kSoftmaxWarps);
     bars->abort = 0;
     bars->last = 0;
     fence_mbar_init();
@@ -519,7 +541,19 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     if (t_stage >= 0) pre = min(pre, t_stage - t_begin);
   }
   int issued = 0;
+  const bool stage_here = works && st_hi > st_lo;
+  GroupStager stg;
+  if (warp >= 4 && stage_here) {
+    stg.load(p, b, kvh, row0, P, st_lo, st_hi, threadIdx.x - 128, 0);
+    __syncwarp();
+    if (lane == 0) mbar_arrive_relaxed(&bars->stage_issued);
+  }
   if ((warp == 0 || warp == 2) && works) {
+    if (stage_here) {
+      // a timeout sets the abort flag; the ring loop below then returns early
+      if (lane == 0) wait_bar(&bars->stage_issued, 0, bars, p.err);
+      __syncwarp();
+    }
     const bool is_k = warp == 0;
     if (is_k) {
       if (lane == 0) {
@@ -632,11 +666,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
       }
     } else if (warp == 3) {
-      // ======================= staging of the block's own K/V =======================
-      if (st_hi > st_lo) {
-        WarpStager::run(p, b, kvh, row0, P, st_lo, st_hi, lane);
-        if (lane == 0) mbar_arrive(&bars->staged);
-      }
       // ======================= cluster merge: K ring hand-off =======================
       // Once this CTA's last Q*K^T has completed no copy or MMA touches its K
       // ring again: tell the other splits they may write their rows into it.
@@ -654,6 +683,12 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     // Both groups work on every key tile: group g takes its keys
     // [64g, 64g + 64) with a running max / sum of its own and accumulates
     // into O_g; the two partial softmaxes are merged per row at the end.
+    // ---- staging of the block's own K/V (first round loaded before the rings) ----
+    if (stage_here) {
+      stg.finish(p, b, kvh, row0, P, st_lo, st_hi, threadIdx.x - 128);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->staged);
+    }
     const int grp = (warp - 4) >> 2;
     const int wq = warp & 3;
     const int m = wq * 32 + lane;                   // packed row = TMEM lane
