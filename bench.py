@@ -686,6 +686,132 @@ def run_select(args):
         dist.destroy_process_group()
 
 
+REORDER_LABELS = {
+    "reorder_serving": "reorder_serving: B64 token rows of up to 2048 (context length, Table 1), "
+                       "lengths ~U[512,2048], per-sequence mask fraction ~U(0.1,0.9)",
+}
+
+
+def run_reorder(args):
+    """Reordering + restoration (Sec. 5.1 steps 2/4, Sec. 5.2 steps 1/8): one
+    step = zarya_reorder of a batch of token rows, then zarya_restore of the
+    reordered rows. Stable form (Mode B) in `value`; the keyed form (Mode A's
+    token shuffling) alongside."""
+    import torch
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    zbuild.build()
+    from paper_2609_19868_gb300 import _binding as zb
+    from paper_2609_19868_gb300 import workloads as wl
+
+    zb.load()
+    zb.check_device_error()
+    name = "reorder_serving"
+    w = wl.make_reorder(name, seed=wl.REORDER_SPECS[name]["seed"] + 1000 * rank)
+    stream = torch.cuda.Stream(dev)
+    B, L = w.B, w.max_len
+    t = torch.as_tensor(w.tokens).to(dev)
+    m = torch.as_tensor(w.is_masked).to(dev)
+    k = torch.as_tensor(w.order_key.view(np.int32)).to(dev)
+    ln = torch.as_tensor(w.lens).to(dev)
+    perm, out, back = (torch.empty_like(t) for _ in range(3))
+    nv = torch.empty(B, dtype=torch.int32, device=dev)
+
+    def step(keyed):
+        zb.reorder(t, m, ln, perm, out, nv, order_key=k if keyed else None, stream=stream)
+        zb.restore(out, perm, ln, back, stream=stream)
+
+    K, W = args.steps, args.warmup
+    res = {}
+    for keyed in (False, True):
+        with torch.cuda.stream(stream):
+            for _ in range(W):
+                step(keyed)
+        torch.cuda.synchronize()
+        assert zb.check_device_error(stream) == 0
+        g = torch.cuda.CUDAGraph()
+        per = 20
+        with torch.cuda.graph(g, stream=stream):
+            for _ in range(per):
+                step(keyed)
+        g.replay()
+        torch.cuda.synchronize()
+        reps = max(1, K // per)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        res[keyed] = e0.elapsed_time(e1) / (reps * per)
+    assert np.array_equal(back.cpu().numpy(), w.tokens)
+    ms = res[False]
+    # algorithmic bytes: reorder reads tokens + mask, writes perm + tokens;
+    # restore reads tokens + perm, writes tokens (4-byte ints, 1-byte mask)
+    n_pos = int(w.lens.sum())
+    nbytes = n_pos * (4 + 1 + 4 + 4 + 4 + 4 + 4)
+    hbm_peak, _, peak_src = read_peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    # e2e: tokens and mask copied in, restored tokens copied back, every step
+    ht, hm, hb = t.cpu().pin_memory(), m.cpu().pin_memory(), torch.empty_like(t, device="cpu").pin_memory()
+
+    def e2e_step():
+        t.copy_(ht, non_blocking=True)
+        m.copy_(hm, non_blocking=True)
+        step(False)
+        hb.copy_(back, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(W):
+            e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n_e2e = min(K, 500)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(n_e2e):
+            e2e_step()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / n_e2e
+    line = {
+        "metric": "reorder + restore steps/s (a batch of token rows reordered visible-first, "
+                  "then restored)",
+        "value": round(1e3 / ms, 2), "unit": "steps/s", "n_gpus": 1, "steps": K, "warmup": W,
+        "ms_per_step": round(ms, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int32", "data": "synthetic (seeded token ids and masks)",
+        "config": {"workload": REORDER_LABELS[name], "global_batch": B,
+                   "keyed_ms_per_step": round(res[True], 5),
+                   "launch": "CUDA graphs of 20 steps (programmatic dependent launch)",
+                   "l2": "inputs resident (1.6 MB); latency-bound"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": None,
+                     "kernel": "reorder_kernel + restore_kernel (launch-latency bound)",
+                     "algorithmic_bytes": nbytes, "peak_source": f"{peak_src} HBM copy bandwidth"},
+        "e2e": {"value": round(1e3 / e2e_ms, 2), "unit": "steps/s",
+                "h2d_bytes_per_step": int(t.numel() * 4 + m.numel()),
+                "d2h_bytes_per_step": int(back.numel() * 4)},
+        "gpu_launches": 2 * K,
+    }
+    if not args.no_cpu_baseline:
+        from oracle import reorder as ro
+
+        nb = 8
+        t0 = time.perf_counter()
+        p_, o_, _ = ro.reorder(w.tokens[:nb], w.is_masked[:nb], w.lens[:nb])
+        ro.restore(o_, p_, w.lens[:nb])
+        dt = (time.perf_counter() - t0) * B / nb
+        line["cpu_baseline"] = {"value": round(1.0 / dt, 4), "unit": "steps/s", "cores": 1,
+                                "kind": "oracle",
+                                "sample": f"{nb} of {B} sequences (python oracle), scaled"}
+    print(json.dumps(line), flush=True)
+
+
 def _oracle_select_rows(w, T, n_draft, n_verify, vtokens):
     """The sampling oracle over the first n_draft draft rows and n_verify
     verification rows (the per-row work dominates; the per-sequence rules are
@@ -879,7 +1005,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=None,
                     choices=list(WORKLOAD_LABELS) + list(SELECT_LABELS))
-    ap.add_argument("--path", choices=["attention", "select"], default="attention",
+    ap.add_argument("--path", choices=["attention", "select", "reorder"], default="attention",
                     help="attention: the slot-decode layer step (stage + attention + commit); "
                          "select: slot selection + token acceptance over logits")
     ap.add_argument("--temperature", type=float, default=0.0)
@@ -891,7 +1017,14 @@ def main():
         args.warmup = 3
     if args.workload is None:
         args.workload = "select_decode_small" if args.path == "select" else "decode_small"
-    if args.path == "select":
+    if args.path == "reorder":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable":
+                              "the reorder path's reference arm is its oracle, timed as "
+                              "cpu_baseline in the --path reorder line"}), flush=True)
+        else:
+            run_reorder(args)
+    elif args.path == "select":
         if args.impl == "reference":
             run_select_reference(args)
         else:

@@ -80,6 +80,7 @@ typedef enum { ZARYA_BF16 = 0, ZARYA_FP32 = 1 } zarya_dtype;
 #define ZARYA_DEVERR_TIMEOUT 5        /* a pipeline wait gave up (no progress for ~2 s) */
 #define ZARYA_DEVERR_MASK_MODE 6      /* mask_mode[b] not a zarya_mask_mode */
 #define ZARYA_DEVERR_TOKEN 7          /* a verification token outside [0, vocab) */
+#define ZARYA_DEVERR_PERM 8           /* a permutation entry outside [0, lens[b]) */
 
 /* Shapes and host-known bounds shared by both calls. */
 typedef struct {
@@ -338,6 +339,49 @@ zarya_status zarya_verify_accept(const void* logits, const int32_t* tokens,
                                  const int32_t* n_slots, const int32_t* slot_len,
                                  float* token_prob, int32_t* slot_accept, int32_t* accept_len,
                                  const zarya_sample_desc* desc, zarya_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Reordering and restoration (Sec. 5.1 steps 2 and 4, Sec. 5.2 steps 1 and 8).
+ *
+ * Before the first forward pass a sequence is reordered so that every
+ * unmasked (visible) token comes before every masked one; after the last
+ * step it is restored to the original order. Sequences are the rows of
+ * [batch, max_len] arrays: sequence b's tokens are its first lens[b]
+ * positions (0 <= lens[b] <= max_len; otherwise ZARYA_DEVERR_ROWS and the
+ * sequence is treated as empty). Positions at or past lens[b] are copied
+ * through unchanged and get perm -1.
+ */
+
+/*
+ * perm[b, i] = the original position of reordered position i: the unmasked
+ * positions in their order, then the masked positions in their order or,
+ * when order_key is given, by ascending (order_key, position) (the token
+ * shuffling of Mode A, Table 2). perm doubles as the position ids of the
+ * reordered sequence. tokens_out[b, i] = tokens[b, perm[b, i]];
+ * n_unmasked[b] = the number of unmasked positions (the prefix length of the
+ * reordered sequence).
+ *  tokens     [batch, max_len] int32 (read)
+ *  is_masked  [batch, max_len] uint8 (read; nonzero = masked)
+ *  order_key  [batch, max_len] uint32 (read) or NULL
+ *  lens       [batch] int32 (read)
+ *  perm, tokens_out [batch, max_len] int32 (written; tokens_out must not
+ *             overlap tokens)
+ *  n_unmasked [batch] int32 (written)
+ */
+zarya_status zarya_reorder(const int32_t* tokens, const uint8_t* is_masked,
+                           const uint32_t* order_key, const int32_t* lens, int32_t batch,
+                           int32_t max_len, int32_t* perm, int32_t* tokens_out,
+                           int32_t* n_unmasked, zarya_stream_t stream);
+
+/*
+ * tokens_out[b, perm[b, i]] = tokens[b, i] for i < lens[b] (perm as written
+ * by zarya_reorder); positions past lens[b] copied through. A perm entry
+ * outside [0, lens[b]) sets ZARYA_DEVERR_PERM and is skipped. tokens_out
+ * must not overlap tokens.
+ */
+zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int32_t* lens,
+                           int32_t batch, int32_t max_len, int32_t* tokens_out,
+                           zarya_stream_t stream);
 
 /*
  * Synchronises `stream`, then reads and clears the error word of the device

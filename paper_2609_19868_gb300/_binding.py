@@ -102,6 +102,10 @@ def load() -> ctypes.CDLL:
     lib.zarya_kv_append_commit_to.restype = ctypes.c_int
     lib.zarya_kv_commit_staged.argtypes = [vp, vp, vp, dp, vp]
     lib.zarya_kv_commit_staged.restype = ctypes.c_int
+    lib.zarya_reorder.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp, vp]
+    lib.zarya_reorder.restype = ctypes.c_int
+    lib.zarya_restore.argtypes = [vp, vp, vp, i32, i32, vp, vp]
+    lib.zarya_restore.restype = ctypes.c_int
     sp = ctypes.POINTER(SampleDesc)
     lib.zarya_draft_select.argtypes = [vp] * 11 + [sp, vp]
     lib.zarya_draft_select.restype = ctypes.c_int
@@ -295,6 +299,42 @@ def kv_commit_staged(accept_len, cache_lens, new_lens, desc: AttnDesc, stream=No
                                        ctypes.byref(desc), _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_kv_commit_staged")
+
+
+def reorder(tokens, is_masked, lens, perm, tokens_out, n_unmasked, order_key=None,
+            stream=None) -> None:
+    """``zarya_reorder``: unmasked positions first, then masked ones (in order,
+    or by ``order_key``); Sec. 5.1 step 2 / Sec. 5.2 step 1."""
+    _check_cuda("tokens", tokens, torch.int32)
+    _check_cuda("is_masked", is_masked, torch.uint8)
+    _check_cuda("lens", lens, torch.int32)
+    _check_cuda("perm", perm, torch.int32)
+    _check_cuda("tokens_out", tokens_out, torch.int32)
+    _check_cuda("n_unmasked", n_unmasked, torch.int32)
+    if order_key is not None:
+        _check_cuda("order_key", order_key, torch.int32)   # uint32 bits in an int32 tensor
+    B, L = tokens.shape
+    for name, t in (("is_masked", is_masked), ("perm", perm), ("tokens_out", tokens_out)):
+        if tuple(t.shape) != (B, L):
+            raise ValueError(f"{name} must be [{B}, {L}]")
+    st = load().zarya_reorder(_ptr(tokens), _ptr(is_masked), _ptr(order_key), _ptr(lens), B, L,
+                              _ptr(perm), _ptr(tokens_out), _ptr(n_unmasked), _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_reorder")
+
+
+def restore(tokens, perm, lens, tokens_out, stream=None) -> None:
+    """``zarya_restore``: back to the original order (Sec. 5.1 step 4 / Sec. 5.2
+    step 8)."""
+    _check_cuda("tokens", tokens, torch.int32)
+    _check_cuda("perm", perm, torch.int32)
+    _check_cuda("lens", lens, torch.int32)
+    _check_cuda("tokens_out", tokens_out, torch.int32)
+    B, L = tokens.shape
+    st = load().zarya_restore(_ptr(tokens), _ptr(perm), _ptr(lens), B, L, _ptr(tokens_out),
+                              _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_restore")
 
 
 def make_sample_desc(*, batch: int, vocab: int, dtype: int, max_slots: int, total_rows: int,

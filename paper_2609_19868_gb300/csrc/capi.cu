@@ -525,6 +525,56 @@ zarya_status zarya_kv_commit_staged(const int32_t* accept_len, const int32_t* ca
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the commit kernel", ce);
 }
 
+zarya_status zarya_reorder(const int32_t* tokens, const uint8_t* is_masked,
+                           const uint32_t* order_key, const int32_t* lens, int32_t batch,
+                           int32_t max_len, int32_t* perm, int32_t* tokens_out,
+                           int32_t* n_unmasked, zarya_stream_t stream_) {
+  if (!tokens || !is_masked || !lens || !perm || !tokens_out || !n_unmasked)
+    return ZARYA_ERR_INVALID_ARG;
+  if (batch < 1 || max_len < 1 || static_cast<const void*>(tokens_out) == tokens)
+    return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, tokens);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  ReorderParams p{};
+  p.tokens = tokens;
+  p.is_masked = is_masked;
+  p.order_key = order_key;
+  p.lens = lens;
+  p.perm = perm;
+  p.tokens_out = tokens_out;
+  p.n_unmasked = n_unmasked;
+  p.err = err;
+  p.B = batch;
+  p.max_len = max_len;
+  ce = launch_reorder(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the reorder kernel", ce);
+}
+
+zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int32_t* lens,
+                           int32_t batch, int32_t max_len, int32_t* tokens_out,
+                           zarya_stream_t stream_) {
+  if (!tokens || !perm || !lens || !tokens_out) return ZARYA_ERR_INVALID_ARG;
+  if (batch < 1 || max_len < 1 || tokens_out == tokens) return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, tokens);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  ReorderParams p{};
+  p.tokens = tokens;
+  p.perm_in = perm;
+  p.lens = lens;
+  p.tokens_out = tokens_out;
+  p.err = err;
+  p.B = batch;
+  p.max_len = max_len;
+  ce = launch_restore(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the restore kernel", ce);
+}
+
 zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {
   if (code) *code = 0;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);

@@ -351,3 +351,44 @@ def make_sampling(name: str, device="cpu", seed: Optional[int] = None,
                             slot_len=i32(L), row_offsets=i32(offs), draft_logits=draft,
                             n_verify=i32(n_ver), verify_offsets=i32(voffs),
                             verify_tokens=i32(v_tok), verify_logits=verify)
+
+
+# --------------------------------------------------------------------------
+# Token rows for reordering / restoration (Sec. 5.1 steps 2/4, Sec. 5.2
+# steps 1/8). Recipe (rng = numpy.random.default_rng(seed), in this order):
+# sequence lengths ~ U{lo..max_len}; per sequence a mask fraction ~ U(0.1,
+# 0.9) and per position a Bernoulli draw with it (masked positions scattered,
+# as in Mode A's first-hitting sampling or fill-in-the-middle prompts);
+# token ids ~ U{0..V-1}; order keys ~ U{0..2^32-1} (Mode A's token shuffling).
+# max_len 2048 is the models' context length (Table 1).
+
+REORDER_SPECS = {
+    "reorder_small": dict(seed=30, B=4, max_len=300, lo=1),
+    "reorder_serving": dict(seed=31, B=64, max_len=2048, lo=512),
+}
+
+
+@dataclass
+class ReorderWorkload:
+    name: str
+    B: int
+    max_len: int
+    lens: np.ndarray        # int32 [B]
+    tokens: np.ndarray      # int32 [B, max_len]
+    is_masked: np.ndarray   # uint8 [B, max_len]
+    order_key: np.ndarray   # uint32 [B, max_len]
+
+
+def make_reorder(name: str, seed: Optional[int] = None) -> ReorderWorkload:
+    spec = dict(REORDER_SPECS[name])
+    if seed is not None:
+        spec["seed"] = seed
+    rng = np.random.default_rng(spec["seed"])
+    B, L = spec["B"], spec["max_len"]
+    lens = rng.integers(spec["lo"], L + 1, size=B).astype(np.int32)
+    frac = rng.uniform(0.1, 0.9, size=(B, 1))
+    mask = (rng.random((B, L)) < frac).astype(np.uint8)
+    tokens = rng.integers(0, QWEN3_VOCAB, size=(B, L)).astype(np.int32)
+    key = rng.integers(0, 2 ** 32, size=(B, L), dtype=np.uint64).astype(np.uint32)
+    return ReorderWorkload(name=name, B=B, max_len=L, lens=lens, tokens=tokens,
+                           is_masked=mask, order_key=key)

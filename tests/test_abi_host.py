@@ -235,3 +235,21 @@ def test_sampling_rejects_null_and_misaligned_pointers(lib):
     assert _verify(lib, _sdesc(), tokens=None) == 1
     assert _verify(lib, _sdesc(), logits=FAKE + 4) == 1
     assert _draft(lib, _sdesc(batch=65536, max_slots=65536)) == 2
+
+
+def test_reorder_restore_reject_invalid_calls(lib):
+    vp = ctypes.c_void_p
+
+    def reo(tokens=FAKE, out=FAKE + 64, batch=2, max_len=8, mask=FAKE):
+        return lib.zarya_reorder(vp(tokens), vp(mask), vp(None), vp(FAKE), batch, max_len,
+                                 vp(FAKE), vp(out), vp(FAKE), None)
+
+    assert reo(tokens=None) == 1
+    assert reo(mask=None) == 1
+    assert reo(out=None) == 1
+    assert reo(out=FAKE) == 1            # in place is refused
+    assert reo(batch=0) == 1
+    assert reo(max_len=0) == 1
+    assert lib.zarya_restore(vp(FAKE), vp(None), vp(FAKE), 2, 8, vp(FAKE + 64), None) == 1
+    assert lib.zarya_restore(vp(FAKE), vp(FAKE), vp(FAKE), 2, 8, vp(FAKE), None) == 1
+    assert lib.zarya_restore(vp(FAKE), vp(FAKE), vp(FAKE), 0, 8, vp(FAKE + 64), None) == 1
