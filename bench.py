@@ -812,6 +812,116 @@ def run_reorder(args):
     print(json.dumps(line), flush=True)
 
 
+def run_mode_a(args):
+    """Mode A (Sec. 5.1): the mask-budget plan of a batch (once per
+    generation), then per step the draw of every revealed position's token
+    (zarya_sample_rows over those rows' logits). Batch of 64 sequences with 256
+    masked tokens each, T = 64 diffusion steps, alpha_0 = 0.25 (the paper's
+    default): a plan of about 64 + 192 steps revealing one token per sequence
+    at most steps, so a step samples 64 rows of the Qwen3 vocabulary."""
+    import torch
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    zbuild.build()
+    from paper_2609_19868_gb300 import _binding as zb
+    from paper_2609_19868_gb300 import session
+    from paper_2609_19868_gb300 import workloads as wl
+
+    zb.load()
+    zb.check_device_error()
+    B, n_mask, T_steps, a0 = 64, 256, 64, 0.25
+    temp = args.temperature
+    stream = torch.cuda.Stream(dev)
+    nm = torch.full((B,), n_mask, dtype=torch.int32, device=dev)
+    counts = torch.zeros((B, T_steps + n_mask), dtype=torch.int32, device=dev)
+    steps = torch.zeros(B, dtype=torch.int32, device=dev)
+    # logits of one revealed row per sequence (64 rows), rotated copies > L2
+    w = wl.make_sampling("select_decode_small", device=dev)
+    rows = B
+    eb = 2
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    n_rot = max(2, math.ceil(3 * l2 / (rows * w.V * eb)))
+    src = w.draft_logits[:rows]
+    rots = []
+    for r in range(n_rot):
+        sw = wl.SamplingWorkload(name="mode_a", B=rows, V=w.V, dtype="bf16",
+                                 n_slots=np.ones(rows, dtype=np.int32),
+                                 slot_len=np.ones(rows, dtype=np.int32),
+                                 row_offsets=np.arange(rows + 1, dtype=np.int32),
+                                 draft_logits=src.roll(r, 0), n_verify=np.ones(rows, dtype=np.int32),
+                                 verify_offsets=np.arange(rows + 1, dtype=np.int32),
+                                 verify_tokens=np.zeros(rows, dtype=np.int32),
+                                 verify_logits=src[:1])
+        rots.append(session.upload_sampling(sw, dev, temperature=temp, seed=9, offset=r))
+    K, W = args.steps, args.warmup
+
+    def plan():
+        zb.mode_a_budget(nm, T_steps, a0, 9, 0, counts, steps, stream=stream)
+
+    def sample(sb):
+        zb.sample_rows(sb.draft_logits, sb.draft_tokens, sb.draft_prob, sb.draft_desc,
+                       stream=stream)
+
+    def timed(fn_graph, reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                fn_graph.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    with torch.cuda.stream(stream):
+        for i in range(max(W, n_rot)):
+            plan()
+            sample(rots[i % n_rot])
+    torch.cuda.synchronize()
+    assert zb.check_device_error(stream) == 0
+    gp = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gp, stream=stream):
+        for _ in range(10):
+            plan()
+    gs = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gs, stream=stream):
+        for sb in rots:
+            sample(sb)
+    gp.replay()
+    gs.replay()
+    torch.cuda.synchronize()
+    plan_ms = timed(gp, max(1, K // 10)) / 10
+    step_ms = timed(gs, max(1, K // n_rot)) / n_rot
+    assert zb.check_device_error(stream) == 0
+    n_steps = steps.cpu().numpy()
+    nbytes = rows * w.V * eb
+    hbm_peak, _, peak_src = read_peaks()
+    gbs = nbytes / (step_ms * 1e-3) / 1e9
+    line = {
+        "metric": "Mode A sampling steps/s (the revealed rows' tokens drawn from their logits)",
+        "value": round(1e3 / step_ms, 2), "unit": "steps/s", "n_gpus": 1, "steps": K,
+        "warmup": W, "ms_per_step": round(step_ms, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32 (bf16 logits)",
+        "data": "synthetic (seeded N(0,2^2) logits with peaked tokens)",
+        "config": {"workload": f"mode_a: B{B}, {n_mask} masked tokens, T={T_steps}, alpha_0={a0}, "
+                               f"{rows} revealed rows per step, V {w.V}",
+                   "temperature": temp,
+                   "plan_ms": round(plan_ms, 5),
+                   "plan_steps_mean": float(n_steps.mean()),
+                   "l2": f"{n_rot} rotating logits copies (> L2 between reuses)"},
+        "roofline": {"bound": "hbm" if temp == 0 else "alu", "achieved": round(gbs, 1),
+                     "peak": hbm_peak, "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
+                     "traffic": None, "kernel": "row_pass_kernel (zarya_sample_rows)",
+                     "algorithmic_bytes": nbytes, "peak_source": f"{peak_src} HBM copy bandwidth"},
+        "e2e": None,
+        "gpu_launches": K,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def _oracle_select_rows(w, T, n_draft, n_verify, vtokens):
     """The sampling oracle over the first n_draft draft rows and n_verify
     verification rows (the per-row work dominates; the per-sequence rules are
@@ -1005,7 +1115,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=None,
                     choices=list(WORKLOAD_LABELS) + list(SELECT_LABELS))
-    ap.add_argument("--path", choices=["attention", "select", "reorder"], default="attention",
+    ap.add_argument("--path", choices=["attention", "select", "reorder", "mode_a"],
+                    default="attention",
                     help="attention: the slot-decode layer step (stage + attention + commit); "
                          "select: slot selection + token acceptance over logits")
     ap.add_argument("--temperature", type=float, default=0.0)
@@ -1017,7 +1128,13 @@ def main():
         args.warmup = 3
     if args.workload is None:
         args.workload = "select_decode_small" if args.path == "select" else "decode_small"
-    if args.path == "reorder":
+    if args.path == "mode_a":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable":
+                              "the Mode A path is measured against its roofline only"}), flush=True)
+        else:
+            run_mode_a(args)
+    elif args.path == "reorder":
         if args.impl == "reference":
             print(json.dumps({"impl": "reference", "unavailable":
                               "the reorder path's reference arm is its oracle, timed as "

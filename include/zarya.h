@@ -340,6 +340,40 @@ zarya_status zarya_verify_accept(const void* logits, const int32_t* tokens,
                                  float* token_prob, int32_t* slot_accept, int32_t* accept_len,
                                  const zarya_sample_desc* desc, zarya_stream_t stream);
 
+/*
+ * Steps 3-4 of either mode without the selection: the draw and its
+ * probability for every row of the sequences in desc->row_offsets (row r of
+ * [row_offsets[0], row_offsets[B])), as defined above (argmax at T = 0,
+ * Gumbel-max over the Philox noise at T > 0). In Mode A these are the rows of
+ * the positions a step reveals (Sec. 5.1 step 3). n_slots / slot_len and the
+ * thresholds of desc are not used.
+ *  tokens [total_rows] int32, prob [total_rows] float (written for those rows)
+ */
+zarya_status zarya_sample_rows(const void* logits, int32_t* tokens, float* prob,
+                               const zarya_sample_desc* desc, zarya_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Mode A mask-budget planning (Sec. 5.1 step 1).
+ *
+ * For sequence b with n = n_masked[b] masked tokens: with T > 0, exactly T
+ * diffusion steps reveal Binomial(n, alpha0) of them, diffusion step s (of T)
+ * revealing Binomial(r_s, 1 / (T - s)) of the r_s not yet revealed (the last
+ * takes the rest), and the remaining n - n_diff tokens are revealed one per
+ * step after them; with T = 0 the noise is ignored: ceil(n / 4) steps of 4
+ * (the last takes the remainder); n = 0 gives no step. Each binomial draw is
+ * the sum of Bernoulli trials [u_i < p] (p in fp32) with u_i the uniform
+ * defined above, from Philox4x32-10 with key (seed low, seed high) and counter
+ * (i / 4, b, draw, offset low word), word i % 4; draw 0 is the diffusion
+ * total, draw 1 + s diffusion step s.
+ *  n_masked [batch] int32 (read; negative sets ZARYA_DEVERR_ROWS)
+ *  counts   [batch, max_steps] int32 (written: reveal count of each step, 0 after the plan)
+ *  n_steps  [batch] int32 (written; 0 with ZARYA_DEVERR_ROWS when the plan has more than
+ *           max_steps steps)
+ */
+zarya_status zarya_mode_a_budget(const int32_t* n_masked, int32_t batch, int32_t T, float alpha0,
+                                 uint64_t seed, uint64_t offset, int32_t max_steps,
+                                 int32_t* counts, int32_t* n_steps, zarya_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Reordering and restoration (Sec. 5.1 steps 2 and 4, Sec. 5.2 steps 1 and 8).
  *

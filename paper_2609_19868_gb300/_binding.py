@@ -102,6 +102,11 @@ def load() -> ctypes.CDLL:
     lib.zarya_kv_append_commit_to.restype = ctypes.c_int
     lib.zarya_kv_commit_staged.argtypes = [vp, vp, vp, dp, vp]
     lib.zarya_kv_commit_staged.restype = ctypes.c_int
+    lib.zarya_sample_rows.argtypes = [vp, vp, vp, ctypes.POINTER(SampleDesc), vp]
+    lib.zarya_sample_rows.restype = ctypes.c_int
+    lib.zarya_mode_a_budget.argtypes = [vp, i32, i32, ctypes.c_float, ctypes.c_uint64,
+                                        ctypes.c_uint64, i32, vp, vp, vp]
+    lib.zarya_mode_a_budget.restype = ctypes.c_int
     lib.zarya_reorder.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp, vp]
     lib.zarya_reorder.restype = ctypes.c_int
     lib.zarya_restore.argtypes = [vp, vp, vp, i32, i32, vp, vp]
@@ -299,6 +304,36 @@ def kv_commit_staged(accept_len, cache_lens, new_lens, desc: AttnDesc, stream=No
                                        ctypes.byref(desc), _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_kv_commit_staged")
+
+
+def sample_rows(logits, tokens, prob, desc: SampleDesc, stream=None) -> None:
+    """``zarya_sample_rows``: the draw and its probability for every row in
+    desc.row_offsets (Sec. 5.1 step 3, Sec. 5.2 steps 3-4)."""
+    _check_logits(logits, desc)
+    _check_cuda("tokens", tokens, torch.int32)
+    _check_cuda("prob", prob, torch.float32)
+    st = load().zarya_sample_rows(_ptr(logits), _ptr(tokens), _ptr(prob), ctypes.byref(desc),
+                                  _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_sample_rows")
+
+
+def mode_a_budget(n_masked, T: int, alpha0: float, seed: int, offset: int, counts, n_steps,
+                  stream=None) -> None:
+    """``zarya_mode_a_budget``: per-step reveal counts of Mode A (Sec. 5.1
+    step 1) into counts [B, max_steps] and n_steps [B]."""
+    _check_cuda("n_masked", n_masked, torch.int32)
+    _check_cuda("counts", counts, torch.int32)
+    _check_cuda("n_steps", n_steps, torch.int32)
+    B = n_masked.shape[0]
+    if counts.dim() != 2 or counts.shape[0] != B:
+        raise ValueError("counts must be [B, max_steps]")
+    st = load().zarya_mode_a_budget(_ptr(n_masked), B, int(T), float(alpha0),
+                                    int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+                                    counts.shape[1], _ptr(counts), _ptr(n_steps),
+                                    _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_mode_a_budget")
 
 
 def reorder(tokens, is_masked, lens, perm, tokens_out, n_unmasked, order_key=None,

@@ -525,6 +525,49 @@ zarya_status zarya_kv_commit_staged(const int32_t* accept_len, const int32_t* ca
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the commit kernel", ce);
 }
 
+zarya_status zarya_sample_rows(const void* logits, int32_t* tokens, float* prob,
+                               const zarya_sample_desc* desc, zarya_stream_t stream_) {
+  zarya_status st = check_sample_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!logits || !tokens || !prob || !aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, logits);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  const SampleCall c{logits, nullptr, nullptr, desc, sm_count()};
+  ce = launch_sample_rows(c, tokens, prob, err, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the row-sampling kernel", ce);
+}
+
+zarya_status zarya_mode_a_budget(const int32_t* n_masked, int32_t batch, int32_t T, float alpha0,
+                                 uint64_t seed, uint64_t offset, int32_t max_steps,
+                                 int32_t* counts, int32_t* n_steps, zarya_stream_t stream_) {
+  if (!n_masked || !counts || !n_steps || batch < 1 || max_steps < 1 || T < 0)
+    return ZARYA_ERR_INVALID_ARG;
+  if (!(alpha0 >= 0.f && alpha0 <= 1.f)) return ZARYA_ERR_INVALID_ARG;
+  if (static_cast<long long>(batch) * max_steps > 0x7fffffffLL) return ZARYA_ERR_UNSUPPORTED;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, n_masked);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  ModeAParams p{};
+  p.n_masked = n_masked;
+  p.counts = counts;
+  p.n_steps = n_steps;
+  p.err = err;
+  p.B = batch;
+  p.T = T;
+  p.max_steps = max_steps;
+  p.alpha0 = alpha0;
+  p.key0 = static_cast<uint32_t>(seed);
+  p.key1 = static_cast<uint32_t>(seed >> 32);
+  p.ctr3 = static_cast<uint32_t>(offset);
+  ce = launch_mode_a_budget(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the budget kernel", ce);
+}
+
 zarya_status zarya_reorder(const int32_t* tokens, const uint8_t* is_masked,
                            const uint32_t* order_key, const int32_t* lens, int32_t batch,
                            int32_t max_len, int32_t* perm, int32_t* tokens_out,

@@ -26,6 +26,7 @@
 #include <cstdint>
 
 #include "internal.cuh"
+#include "philox.cuh"
 #include "ptx.cuh"
 
 namespace zarya {
@@ -89,29 +90,10 @@ __device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
   return r;
 }
 
-// Philox4x32 with 10 rounds (Salmon et al., SC'11): each round multiplies
-// counter words 0 and 2 by the round constants into 64-bit products and
-// forms (hi1 ^ c1 ^ k0, lo1, hi0 ^ c3 ^ k1, lo0); the key advances by the
-// Weyl increments between rounds.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r > 0) {
-      k0 += 0x9E3779B9u;
-      k1 += 0xBB67AE85u;
-    }
-    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-  }
-  return c;
-}
-
-// Standard Gumbel variate from one 32-bit draw: u = fl32(fl32(w) 2^-32 +
-// 2^-33) in (0, 1] (the product is exact, so the fma rounds once, like the
-// separate add), E = -log1p(-u) exponential, g = -log(E).
+// Standard Gumbel variate from one 32-bit draw: u in (0, 1] (see
+// uniform_from_word), E = -log1p(-u) exponential, g = -log(E).
 __device__ __forceinline__ float gumbel_from_word(uint32_t w) {
-  const float u = fmaf(__uint2float_rn(w), 0x1p-32f, 0x1p-33f);
+  const float u = uniform_from_word(w);
   const float e = -log1pf(-u);
   return -__logf(e);
 }
@@ -809,6 +791,20 @@ cudaError_t launch_draft_select(const SampleCall& c, const DraftOutputs& o, int*
   s.slot_threshold = c.desc->slot_threshold;
   PdlLaunch l(dim3(1), dim3(kSelectThreads), 0, stream);
   return cudaLaunchKernelEx(&l.cfg, select_kernel, s);
+}
+
+cudaError_t launch_sample_rows(const SampleCall& c, int32_t* tokens, float* prob, int* err,
+                               cudaStream_t stream) {
+  RowArgs a = row_args(c, err);
+  a.out_token = tokens;
+  a.out_prob = prob;
+  const bool bf16 = c.desc->dtype == ZARYA_BF16;
+  const bool gumbel = c.desc->temperature > 0.f;
+  if (bf16)
+    return gumbel ? launch_row_pass<uint16_t, kDraftGumbel>(a, stream)
+                  : launch_row_pass<uint16_t, kDraftArgmax>(a, stream);
+  return gumbel ? launch_row_pass<float, kDraftGumbel>(a, stream)
+                : launch_row_pass<float, kDraftArgmax>(a, stream);
 }
 
 cudaError_t launch_verify_accept(const SampleCall& c, const int32_t* tokens, float* token_prob,

@@ -253,3 +253,23 @@ def test_reorder_restore_reject_invalid_calls(lib):
     assert lib.zarya_restore(vp(FAKE), vp(None), vp(FAKE), 2, 8, vp(FAKE + 64), None) == 1
     assert lib.zarya_restore(vp(FAKE), vp(FAKE), vp(FAKE), 2, 8, vp(FAKE), None) == 1
     assert lib.zarya_restore(vp(FAKE), vp(FAKE), vp(FAKE), 0, 8, vp(FAKE + 64), None) == 1
+
+
+def test_mode_a_budget_and_sample_rows_reject_invalid_calls(lib):
+    vp = ctypes.c_void_p
+
+    def bud(n=FAKE, batch=2, T=4, a0=0.25, max_steps=8, counts=FAKE, steps=FAKE):
+        return lib.zarya_mode_a_budget(vp(n), batch, T, a0, 1, 0, max_steps, vp(counts),
+                                       vp(steps), None)
+
+    assert bud(n=None) == 1
+    assert bud(counts=None) == 1
+    assert bud(steps=None) == 1
+    assert bud(batch=0) == 1
+    assert bud(max_steps=0) == 1
+    assert bud(T=-1) == 1
+    assert bud(a0=1.5) == 1
+    assert bud(a0=float("nan")) == 1
+    assert lib.zarya_sample_rows(vp(None), vp(FAKE), vp(FAKE), ctypes.byref(_sdesc()), None) == 1
+    assert lib.zarya_sample_rows(vp(FAKE), vp(None), vp(FAKE), ctypes.byref(_sdesc()), None) == 1
+    assert lib.zarya_sample_rows(vp(FAKE), vp(FAKE), vp(FAKE), None, None) == 1
