@@ -291,11 +291,18 @@ def run_ours(args):
             fn()
         return g
 
+    def step_copy(db):
+        # the same step with the commit copying the accepted rows again
+        db.stage_and_attend(stream)
+        db.commit(stream, new_lens=lens_next[id(db)])
+
     full, tail = divmod(K, n_rot)
     step_graph = capture(step, n_rot)
     step_tail = capture(step, tail) if tail else None
     attn_graph = capture(attend, n_rot)
     attn_tail = capture(attend, tail) if tail else None
+    copy_graph = capture(step_copy, n_rot)
+    copy_tail = capture(step_copy, tail) if tail else None
 
     def run(graph, tail_graph):
         for _ in range(full):
@@ -336,6 +343,13 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = sampler.stop(t0, time.time()) if sampler else None
     assert zb.check_device_error(stream) == 0
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        c0.record(stream)
+        run(copy_graph, copy_tail)
+        c1.record(stream)
+    torch.cuda.synchronize()
+    copy_ms = max_over_ranks(c0.elapsed_time(c1) / K, dev, world)
     attn_ms = max_over_ranks(a0.elapsed_time(a1) / K, dev, world)
     attn_method = (f"{K} attention launches back to back ({n_rot} per CUDA graph, one per cache "
                    "rotation), CUDA events on the launching stream")
@@ -457,6 +471,20 @@ def run_ours(args):
             "unit": "steps/s",
             "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h),
+        },
+        "step_forms": {
+            "commit_staged": {"ms_per_step": round(total_ms / K, 5),
+                              "note": "zarya_slot_attn_staged + zarya_kv_commit_staged (the "
+                                      "accepted rows are already in place: lengths advance)"},
+            "commit_copy": {"ms_per_step": round(copy_ms, 5),
+                            "steps_per_s": round(replica_throughput(K, world, copy_ms * K), 2),
+                            "note": "zarya_slot_attn_staged + zarya_kv_append_commit_to (the "
+                                    "accepted rows copied again)"},
+        },
+        "model_projection": {
+            "note": "context only: one step per layer, attention path alone",
+            "layers_28_steps_per_s": round(value / 28, 2),
+            "layers_36_steps_per_s": round(value / 36, 2),
         },
         "gpu_launches": 2 * K,   # staged attention, commit (length advance)
         "clocks": clocks,

@@ -10,6 +10,7 @@
 #include <cstdio>
 
 #include "internal.cuh"
+#include "token_ops.cuh"
 
 namespace zarya {
 namespace {

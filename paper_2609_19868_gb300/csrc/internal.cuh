@@ -105,41 +105,9 @@ struct DraftOutputs {
 
 cudaError_t launch_draft_select(const SampleCall& c, const DraftOutputs& o, int* err,
                                 cudaStream_t stream);
-cudaError_t launch_sample_rows(const SampleCall& c, int32_t* tokens, float* prob, int* err,
-                               cudaStream_t stream);
 cudaError_t launch_verify_accept(const SampleCall& c, const int32_t* tokens, float* token_prob,
                                  int32_t* slot_accept, int32_t* accept_len, int* err,
                                  cudaStream_t stream);
-
-// Reordering / restoration of [B, max_len] token rows.
-struct ReorderParams {
-  const int32_t* tokens;
-  const uint8_t* is_masked;   // reorder
-  const uint32_t* order_key;  // reorder, optional
-  const int32_t* lens;
-  const int32_t* perm_in;     // restore
-  int32_t* perm;              // reorder
-  int32_t* tokens_out;
-  int32_t* n_unmasked;        // reorder
-  int* err;
-  int B, max_len;
-};
-
-cudaError_t launch_reorder(const ReorderParams& p, cudaStream_t stream);
-cudaError_t launch_restore(const ReorderParams& p, cudaStream_t stream);
-
-// Mode A mask-budget planning.
-struct ModeAParams {
-  const int32_t* n_masked;
-  int32_t* counts;     // [B, max_steps]
-  int32_t* n_steps;    // [B]
-  int* err;
-  int B, T, max_steps;
-  float alpha0;
-  uint32_t key0, key1, ctr3;
-};
-
-cudaError_t launch_mode_a_budget(const ModeAParams& p, cudaStream_t stream);
 
 // Dynamic shared memory of the tensor-core kernel.
 size_t tc_smem_bytes();

@@ -17,6 +17,7 @@
 #include <cstdint>
 
 #include "internal.cuh"
+#include "token_ops.cuh"
 #include "ptx.cuh"
 
 namespace zarya {

@@ -26,6 +26,7 @@
 #include <cstdint>
 
 #include "internal.cuh"
+#include "token_ops.cuh"
 #include "philox.cuh"
 #include "ptx.cuh"
 
