@@ -52,6 +52,9 @@ namespace {
 
 constexpr int kThreads = 384;
 constexpr int kSoftmaxWarps = 8;   // warps 4..11: two softmax warpgroups
+// Tiles of K and of V warmed in L2 before the grid dependency wait (all CTAs'
+// first tiles then land before the rest of the ring prefill).
+constexpr int kPrefetchTiles = 2;
 constexpr int kStagesK = 3;
 constexpr int kStagesV = 3;
 constexpr uint32_t kHalfBytes = kBlockN * 64 * 2;   // 128 rows x 128 B
@@ -367,7 +370,7 @@ __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* 
   return true;
 }
 
-// L2 prefetch of the first kStagesK tiles of this CTA's key range (and of its
+// L2 prefetch of the first kPrefetchTiles tiles of this CTA's key range (and of its
 // Q tile when map_q is given), from a reading of the sequence's lengths that
 // may be stale; nothing is prefetched when that reading is out of range.
 __device__ __forceinline__ void prefetch_first_tiles(const CUtensorMap* map_kv,
@@ -388,7 +391,7 @@ __device__ __forceinline__ void prefetch_first_tiles(const CUtensorMap* map_kv,
   const int n_tiles = (kv_end + kBlockN - 1) / kBlockN;
   const int per_split = max(1, (n_tiles + p.splits - 1) / p.splits);
   const int t_begin = split * per_split;
-  const int t_end = min(n_tiles, t_begin + min(per_split, kStagesK));
+  const int t_end = min(n_tiles, t_begin + min(per_split, kPrefetchTiles));
   for (int t = t_begin; t < t_end; ++t) {
     tma_prefetch_l2_4d(map_kv, 0, kvh, t * kBlockN, b);
     tma_prefetch_l2_4d(map_kv, 64, kvh, t * kBlockN, b);
