@@ -93,10 +93,11 @@ struct Plan {
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-// Split-KV plan of the tensor-core path. Work tiles (sequence, KV head,
-// M-tile) whose count already fills the GPU run unsplit; otherwise the key
-// range of each is split so that the slowest CTA (waves x tiles per CTA,
-// plus a fixed per-CTA cost) is as short as possible.
+// Split-KV plan of the tensor-core path: the key range of every work tile
+// (sequence, KV head, M-tile) is split so that the slowest SM (waves x tiles
+// per CTA, plus a fixed per-CTA cost) is as short as possible. Splitting also
+// pays when the tiles already fill the GPU but leave a partial last wave
+// (long_ctx: 512 tiles are 3.4 waves of 152 SMs; two splits make 6.7).
 Plan plan_tc(const zarya_attn_desc* d, int sms) {
   Plan p{};
   p.g = d->n_q_heads / d->n_kv_heads;
@@ -107,7 +108,7 @@ Plan plan_tc(const zarya_attn_desc* d, int sms) {
   int splits = 1;
   if (d->kv_splits > 0) {
     splits = d->kv_splits < tiles ? d->kv_splits : tiles;
-  } else if (p.units < sms) {
+  } else {
     double best = 1e30;
     for (int s = 1; s <= tiles && s <= kMaxClusterSplits; ++s) {
       const long long waves = (p.units * s + sms - 1) / sms;
