@@ -91,12 +91,15 @@ __device__ __forceinline__ __nv_bfloat162 as_bf162(uint32_t w) {
   return r;
 }
 
-// Standard Gumbel variate from one 32-bit draw: u in (0, 1] (see
-// uniform_from_word), E = -log1p(-u) exponential, g = -log(E).
-__device__ __forceinline__ float gumbel_from_word(uint32_t w) {
-  const float u = uniform_from_word(w);
+// Standard Gumbel variate from a uniform u in (0, 1] (see uniform_from_word):
+// E = -log1p(-u) exponential, g = -log(E); g decreases as u grows.
+__device__ __forceinline__ float gumbel_from_uniform(float u) {
   const float e = -log1pf(-u);
   return -__logf(e);
+}
+
+__device__ __forceinline__ float gumbel_from_word(uint32_t w) {
+  return gumbel_from_uniform(uniform_from_word(w));
 }
 
 // Per-thread reduction state of the row pass.
@@ -122,9 +125,29 @@ __device__ __forceinline__ void absorb_max(RowState& st, float vm, float k2) {
   st.m = vm;
 }
 
+// Upper bound of any Gumbel variate gumbel_from_word makes: the smallest u is
+// 2^-33, where E = -log1p(-u) is 2^-33 to within float rounding and
+// g = -log(E) = 33 ln 2 = 22.87; 24 leaves room for the approximate log.
+constexpr float kGumbelMax = 24.0f;
+
+// Floats ordered as ints (for atomicMax on shared memory): non-negative
+// floats keep their bits, negative ones flip all bits but the sign.
+__device__ __forceinline__ int float_order(float f) {
+  const int b = __float_as_int(f);
+  return b >= 0 ? b : b ^ 0x7fffffff;
+}
+__device__ __forceinline__ float order_float(int k) {
+  return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff);
+}
+
+// `bound` (Gumbel form): a score x / T + g that some element of the row
+// reaches; a vector whose largest possible score, fma(max x, 1/T,
+// kGumbelMax), stays below it cannot hold the draw, and skips its noise
+// (its softmax terms are still added).
 template <int kMode, int kN>
 __device__ __forceinline__ void absorb(RowState& st, const float (&x)[kN], int v0,
-                                       const RowArgs& a, uint32_t row) {
+                                       const RowArgs& a, uint32_t row,
+                                       float bound = -INFINITY) {
   float vm = x[0];
 #pragma unroll
   for (int j = 1; j < kN; ++j) vm = fmaxf(vm, x[j]);
@@ -146,6 +169,17 @@ __device__ __forceinline__ void absorb(RowState& st, const float (&x)[kN], int v
     st.s += acc;
   }
   if (kMode == kDraftGumbel) {
+    const float thr = fmaxf(bound, st.bz);
+    if (fmaf(vm, a.inv_t, kGumbelMax) < thr) return;
+    // An element of this vector reaches thr only if its noise exceeds
+    // t = thr - max x / T (less 0.01 for the rounding of the noise and of
+    // the score), i.e. only if E = -log1p(-u) < exp(-t), i.e. only if
+    // u < -expm1(-exp(-t)): larger u skip both logarithms.
+    float u_lim = 2.f;
+    if (thr > -INFINITY) {
+      const float t = thr - vm * a.inv_t - 0.01f;
+      u_lim = -expm1f(-expf(-t));
+    }
     // kN is 4 or 8 with v0 a multiple of 4: one Philox block per 4 elements.
 #pragma unroll
     for (int q = 0; q < kN / 4; ++q) {
@@ -154,7 +188,9 @@ __device__ __forceinline__ void absorb(RowState& st, const float (&x)[kN], int v
       const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const float z = fmaf(x[q * 4 + j], a.inv_t, gumbel_from_word(ws[j]));
+        const float u = uniform_from_word(ws[j]);
+        if (u > u_lim) continue;
+        const float z = fmaf(x[q * 4 + j], a.inv_t, gumbel_from_uniform(u));
         const int v = v0 + q * 4 + j;
         if (z > st.bz || (z == st.bz && v < st.bi)) {
           st.bz = z;
@@ -324,6 +360,7 @@ template <typename TIn, int kMode>
 __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) row_pass_kernel(const RowArgs a) {
   extern __shared__ __align__(128) uint4 stage_buf[];
   __shared__ uint64_t full[kStages], empty[kStages];
+  __shared__ int best_score;   // Gumbel form: the CTA's best score so far (float_order)
   __shared__ RowState red[kConsumerWarps];
   __shared__ RowState cta_state;
   __shared__ int abort_flag;
@@ -335,6 +372,7 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) row_pass_kernel(co
       mbar_init(&empty[st], kConsumerWarps);
     }
     abort_flag = 0;
+    best_score = float_order(-INFINITY);
     fence_mbar_init();
   }
   __syncthreads();
@@ -418,14 +456,21 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) row_pass_kernel(co
       if (lane == 0) mbar_arrive(&empty[sidx]);
       const int e0 = (v_lo + c * kChunkVecs + tid) * kEpv;
       if (kMode == kDraftGumbel) {
+        // The CTA's best score so far lets vectors that cannot win skip the
+        // noise; each warp publishes its best after the stage.
+        const float bound = order_float(*static_cast<volatile int*>(&best_score));
 #pragma unroll
         for (int k = 0; k < kVecsPerThread; ++k) {
           if (tid + k * kConsumers < nv) {
             float x[kEpv];
             widen<TIn>(v[k], x);
-            absorb<kMode>(st, x, e0 + k * kConsumers * kEpv, a, urow);
+            absorb<kMode>(st, x, e0 + k * kConsumers * kEpv, a, urow, bound);
           }
         }
+        float wb = st.bz;
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) wb = fmaxf(wb, __shfl_xor_sync(0xffffffffu, wb, d));
+        if (lane == 0 && wb > bound) atomicMax(&best_score, float_order(wb));
       } else {
         float x[kVecsPerThread][kEpv];
 #pragma unroll
