@@ -570,15 +570,27 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(const SelectArgs
   __shared__ uint32_t s_mask[kSelectThreads];   // selected slots 0..31
   __shared__ int s_warp[kWarps];
   __shared__ int s_carry;
-  grid_dependency_wait();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // The block layout was written before the row pass started (which waited
+  // for it): the first chunk's is read before this kernel's wait for the
+  // row pass's draws.
+  int pre_S = 0, pre_L = 0, pre_lo = 0, pre_hi = 0;
+  if (warp < a.B) {
+    pre_S = a.n_slots[warp];
+    pre_L = a.slot_len[warp];
+    pre_lo = a.row_offsets[warp];
+    pre_hi = a.row_offsets[warp + 1];
+  }
+  grid_dependency_wait();
   if (tid == 0) s_carry = 0;
   for (int b0 = 0; b0 < a.B; b0 += kSelectThreads) {
     const int nb = min(kSelectThreads, a.B - b0);
     for (int i = warp; i < nb; i += kWarps) {
       const int b = b0 + i;
-      const int S = a.n_slots[b], L = a.slot_len[b];
-      const int lo = a.row_offsets[b], hi = a.row_offsets[b + 1];
+      const bool pre = b0 == 0 && i == warp;
+      const int S = pre ? pre_S : a.n_slots[b], L = pre ? pre_L : a.slot_len[b];
+      const int lo = pre ? pre_lo : a.row_offsets[b];
+      const int hi = pre ? pre_hi : a.row_offsets[b + 1];
       const bool ok = S >= 1 && L >= 1 && S <= a.max_slots && lo >= 0 && hi <= a.total_rows &&
                       static_cast<long long>(S) * L == static_cast<long long>(hi) - lo;
       float* conf = a.slot_conf + static_cast<int64_t>(b) * a.max_slots;
@@ -709,12 +721,20 @@ struct AcceptArgs {
 
 // Step 6 acceptance: one warp per sequence.
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const AcceptArgs a) {
-  grid_dependency_wait();
+  // The layout (slot counts, lengths, offsets) was written before the row
+  // pass started, which waited for it: it is read before this kernel's wait
+  // for the row pass's probabilities.
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * (kAcceptThreads / 32) + (threadIdx.x >> 5);
+  int S = 0, L = 0, lo = 0, hi = 0;
+  if (b < a.B) {
+    S = a.n_slots[b];
+    L = a.slot_len[b];
+    lo = a.row_offsets[b];
+    hi = a.row_offsets[b + 1];
+  }
+  grid_dependency_wait();
   if (b >= a.B) return;
-  const int S = a.n_slots[b], L = a.slot_len[b];
-  const int lo = a.row_offsets[b], hi = a.row_offsets[b + 1];
   const bool ok = S >= 0 && L >= 1 && S <= a.max_slots && lo >= 0 && hi <= a.total_rows &&
                   static_cast<long long>(S) * L == static_cast<long long>(hi) - lo;
   int32_t* sa = a.slot_accept + static_cast<int64_t>(b) * a.max_slots;
