@@ -452,3 +452,26 @@ def test_calls_capture_into_a_cuda_graph():
     assert torch.equal(sb.accept_len, first[1])
     assert torch.equal(torch.nan_to_num(sb.token_prob, nan=-1.0),
                        torch.nan_to_num(first[2], nan=-1.0))
+
+
+@pytest.mark.parametrize("T", [0.0, 0.8])
+@pytest.mark.parametrize("rows", [8, 24])
+def test_few_full_vocabulary_rows_split_over_a_cluster(T, rows):
+    """Few rows of the full vocabulary: every row is split over a cluster of
+    CTAs (8 for 8 rows) whose partial maxima, sums and draws merge through
+    distributed shared memory; each row against the oracle."""
+    V = wl.QWEN3_VOCAB
+    rng = np.random.default_rng(rows)
+    x = (rng.standard_normal((rows, V)) * 2).astype(np.float32)
+    for r in range(0, rows, 3):
+        x[r, rng.integers(0, V)] += 15.0
+    xb = torch.as_tensor(x).to(torch.bfloat16)
+    out, err, _ = _direct(xb.float().numpy(), [rows], [1], T=T, seed=21, offset=4,
+                          dtype=torch.bfloat16)
+    assert err == 0
+    xh = xb.float().numpy()
+    near = _check_draws(xh, range(rows), out["draft_tokens"], T, 21, 4)
+    assert near <= 1
+    for g in range(rows):
+        assert _p_close(out["draft_prob"][g],
+                        smp.row_probability(xh[g], int(out["draft_tokens"][g]), T))
