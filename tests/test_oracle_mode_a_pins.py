@@ -90,3 +90,15 @@ def test_batch_plan_padding():
     counts, n_steps = ma.budget([10, 0, 5], 0, 0.25)
     assert counts.tolist() == [[4, 4, 2], [0, 0, 0], [4, 1, 0]]
     assert n_steps.tolist() == [3, 0, 2]
+
+
+def test_bernoulli_trial_is_strict_at_equality():
+    # [u < p]: a trial whose uniform equals p exactly fails
+    u = ma.uniforms(4, 0, 0, 0, 8)
+    p = float(u[0])
+    assert ma.binomial(4, 0, 0, 0, 1, p) == 0
+    above = float(np.nextafter(np.float32(p), np.float32(2)))
+    assert ma.binomial(4, 0, 0, 0, 1, above) == 1
+    # and over several trials the count is the number of uniforms strictly below p
+    p = float(np.sort(u)[4])
+    assert ma.binomial(4, 0, 0, 0, 8, p) == 4
