@@ -6,6 +6,8 @@ bytes. Reduced workloads are compared element by element on every output;
 full-size workloads, in the launch configuration the benchmark uses, on
 sampled rows the oracle computes one by one.
 """
+from dataclasses import replace
+
 import numpy as np
 import pytest
 import torch
@@ -219,3 +221,47 @@ def test_cuda_graph_capture_of_a_step_matches_eager(zs):
     assert zb.check_device_error() == 0
     assert torch.equal(db.out, eager.out)
     assert torch.equal(db.cache_lens, eager.cache_lens)
+
+
+# Ragged batches whose grids take several waves of CTAs (one CTA per SM),
+# compared on every output.
+@pytest.mark.parametrize("name,override", [
+    ("ragged_mid", dict(B=48, prefix=("uniform", 37, 400))),        # distinct lengths
+    ("ragged_mid", dict(B=128, prefix=("uniform", 100, 103))),      # many equal lengths
+    ("ragged_mid", dict(B=129, prefix=("uniform", 37, 150))),
+    ("serving_mix", dict(B=40, prefix=("loguniform", 20, 900))),    # paged, mixed L and masks
+])
+def test_multi_wave_ragged_batch_matches_oracle_everywhere(zs, oracle_mod, name, override):
+    w = wl.make(name, seed=11, **override)
+    db = _run(zs, w)
+    kc, vc = oracle_staged(oracle_mod, w)
+    ref = oracle_full(oracle_mod, w, kc, vc)
+    got = db.out
+    assert not torch.isnan(got).any()
+    ok, err, scale = tolerance_ok(got, ref, w.dtype)
+    assert ok, f"{name} {override}: max|err|={err:.3e} max|ref|={scale:.3f}"
+
+
+def _one_sequence(w, b):
+    """Sequence b of a contiguous-cache workload as a batch of one."""
+    lo, hi = int(w.q_row_offsets[b]), int(w.q_row_offsets[b + 1])
+    sl = slice(b, b + 1)
+    return replace(w, B=1, cache_lens=w.cache_lens[sl].copy(), n_slots=w.n_slots[sl].copy(),
+                   slot_len=w.slot_len[sl].copy(), mask_mode=w.mask_mode[sl].copy(),
+                   accept_len=w.accept_len[sl].copy(),
+                   q_row_offsets=np.array([0, hi - lo], dtype=w.q_row_offsets.dtype),
+                   q=w.q[lo:hi].clone(), k_cache=w.k_cache[sl].clone(),
+                   v_cache=w.v_cache[sl].clone(), k_new=w.k_new[lo:hi].clone(),
+                   v_new=w.v_new[lo:hi].clone())
+
+
+def test_batching_leaves_each_sequence_bitwise_unchanged(zs):
+    """With one split per tile a sequence's outputs are the same bits whether
+    its CTAs run inside a multi-wave batch or alone."""
+    w = wl.make("ragged_mid", seed=13, B=48, prefix=("uniform", 37, 400))
+    full = _run(zs, w, kv_splits=1).out
+    order = np.argsort(-(w.cache_lens.astype(np.int64) + w.R), kind="stable")
+    for b in sorted({int(order[0]), int(order[-1]), 0, 17, 47}):
+        lo, hi = int(w.q_row_offsets[b]), int(w.q_row_offsets[b + 1])
+        alone = _run(zs, _one_sequence(w, b), kv_splits=1).out
+        assert torch.equal(full[lo:hi], alone), f"sequence {b}"
