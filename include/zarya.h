@@ -418,6 +418,24 @@ zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int
                            zarya_stream_t stream);
 
 /*
+ * Moves `bytes` bytes from src to dst with a kernel instead of a copy engine:
+ * a grid of at most 24 CTAs reads and writes 16-byte vectors, reaching host
+ * memory through its device mapping. Each of src and dst is device memory or
+ * page-locked host memory the device can address (cudaHostAlloc /
+ * cudaMallocHost, or cudaHostRegister with the mapped flag; with unified
+ * addressing every page-locked allocation is mapped); at least one is device
+ * memory. Meant for a step's inputs and outputs: inside a CUDA graph the copy
+ * is one more kernel node, with none of the copy-engine hand-over a memcpy
+ * node costs next to kernels. Not a step of the paper's method.
+ *  src, dst: 16-byte aligned, ranges not overlapping; bytes: any (0 launches
+ *            nothing). Ordered on `stream` like any kernel.
+ * Returns ZARYA_ERR_INVALID_ARG (nothing launched) for a NULL or unaligned
+ * pointer, memory the device cannot address, two host buffers, or
+ * overlapping ranges.
+ */
+zarya_status zarya_copy(const void* src, void* dst, size_t bytes, zarya_stream_t stream);
+
+/*
  * Synchronises `stream`, then reads and clears the error word of the device
  * that owns it. Returns ZARYA_OK when it was clear, ZARYA_ERR_DEVICE_FAULT
  * when it was set (*code receives its ZARYA_DEVERR_* value; code may be

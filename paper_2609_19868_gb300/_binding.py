@@ -116,6 +116,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_draft_select.restype = ctypes.c_int
     lib.zarya_verify_accept.argtypes = [vp] * 7 + [sp, vp]
     lib.zarya_verify_accept.restype = ctypes.c_int
+    lib.zarya_copy.argtypes = [vp, vp, sz, vp]
+    lib.zarya_copy.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
     lib.zarya_check_device_error.restype = ctypes.c_int
     lib.zarya_last_error.argtypes = []
@@ -370,6 +372,23 @@ def restore(tokens, perm, lens, tokens_out, stream=None) -> None:
                               _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_restore")
+
+
+def copy(dst: torch.Tensor, src: torch.Tensor, stream=None) -> None:
+    """``zarya_copy``: dst <- src (the same number of bytes) by a kernel; each
+    tensor lives on the device or in pinned host memory, at least one on the
+    device."""
+    for name, t in (("src", src), ("dst", dst)):
+        if not isinstance(t, torch.Tensor) or not (t.is_cuda or t.is_pinned()):
+            raise TypeError(f"{name} must be a CUDA tensor or a pinned host tensor")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+    nbytes = src.numel() * src.element_size()
+    if dst.numel() * dst.element_size() != nbytes:
+        raise ValueError("src and dst differ in size")
+    st = load().zarya_copy(_ptr(src), _ptr(dst), nbytes, _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_copy")
 
 
 def make_sample_desc(*, batch: int, vocab: int, dtype: int, max_slots: int, total_rows: int,

@@ -620,6 +620,43 @@ zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the restore kernel", ce);
 }
 
+// The device address of `p` (device memory as is; page-locked host memory
+// through its mapping), or nullptr when the device cannot address it.
+static const void* device_address(const void* p, bool* is_device) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();   // clear the error the query leaves behind
+    return nullptr;
+  }
+  *is_device = a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+  if (*is_device) return p;
+  if (a.type != cudaMemoryTypeHost) return nullptr;
+  void* d = nullptr;
+  if (cudaHostGetDevicePointer(&d, const_cast<void*>(p), 0) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return d;
+}
+
+zarya_status zarya_copy(const void* src, void* dst, size_t bytes, zarya_stream_t stream_) {
+  if (!src || !dst) return ZARYA_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u)
+    return ZARYA_ERR_INVALID_ARG;
+  if (bytes == 0) return ZARYA_OK;
+  bool src_dev = false, dst_dev = false;
+  const void* s = device_address(src, &src_dev);
+  const void* d = device_address(dst, &dst_dev);
+  if (s == nullptr || d == nullptr || (!src_dev && !dst_dev)) return ZARYA_ERR_INVALID_ARG;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(s), b = reinterpret_cast<uintptr_t>(d);
+  if (a < b + bytes && b < a + bytes) return ZARYA_ERR_INVALID_ARG;   // overlapping ranges
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, src_dev ? src : dst);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  ce = launch_copy(s, const_cast<void*>(d), bytes, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the copy kernel", ce);
+}
+
 zarya_status zarya_check_device_error(zarya_stream_t stream_, int32_t* code) {
   if (code) *code = 0;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);

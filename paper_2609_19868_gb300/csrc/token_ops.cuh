@@ -4,6 +4,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <stddef.h>
 #include <stdint.h>
 
 #include "internal.cuh"
@@ -12,6 +13,10 @@ namespace zarya {
 
 cudaError_t launch_sample_rows(const SampleCall& c, int32_t* tokens, float* prob, int* err,
                                cudaStream_t stream);
+
+// SM copy of `bytes` bytes between device addresses (device memory, or the
+// device mapping of page-locked host memory); src and dst 16-byte aligned.
+cudaError_t launch_copy(const void* src, void* dst, size_t bytes, cudaStream_t stream);
 
 // Reordering / restoration of [B, max_len] token rows.
 struct ReorderParams {

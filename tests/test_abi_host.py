@@ -273,3 +273,20 @@ def test_mode_a_budget_and_sample_rows_reject_invalid_calls(lib):
     assert lib.zarya_sample_rows(vp(None), vp(FAKE), vp(FAKE), ctypes.byref(_sdesc()), None) == 1
     assert lib.zarya_sample_rows(vp(FAKE), vp(None), vp(FAKE), ctypes.byref(_sdesc()), None) == 1
     assert lib.zarya_sample_rows(vp(FAKE), vp(FAKE), vp(FAKE), None, None) == 1
+
+
+def test_copy_rejects_invalid_calls_before_any_cuda_call(lib):
+    vp = ctypes.c_void_p
+    assert lib.zarya_copy(vp(None), vp(FAKE), 64, None) == 1
+    assert lib.zarya_copy(vp(FAKE), vp(None), 64, None) == 1
+    assert lib.zarya_copy(vp(FAKE + 8), vp(FAKE + 4096), 64, None) == 1    # unaligned source
+    assert lib.zarya_copy(vp(FAKE), vp(FAKE + 4100), 64, None) == 1        # unaligned destination
+    assert lib.zarya_copy(vp(FAKE), vp(FAKE + 4096), 0, None) == 0         # nothing to move
+
+
+def test_copy_binding_checks_tensors():
+    import torch
+
+    a = torch.zeros(16, dtype=torch.uint8)
+    with pytest.raises(TypeError):
+        zb.copy(a, a.clone())       # neither pinned nor on a device
