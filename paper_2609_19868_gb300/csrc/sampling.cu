@@ -140,63 +140,52 @@ __device__ __forceinline__ float order_float(int k) {
   return __int_as_float(k >= 0 ? k : k ^ 0x7fffffff);
 }
 
-// `bound` (Gumbel form): a score x / T + g that some element of the row
-// reaches; a vector whose largest possible score, fma(max x, 1/T,
-// kGumbelMax), stays below it cannot hold the draw, and skips its noise
-// (its softmax terms are still added).
-template <int kMode, int kN>
-__device__ __forceinline__ void absorb(RowState& st, const float (&x)[kN], int v0,
-                                       const RowArgs& a, uint32_t row,
-                                       float bound = -INFINITY) {
+// Gumbel selection over one vector of the row (its softmax terms are added
+// by absorb_chunk). `bound` (or the thread's own best, if larger) is a score
+// x / T + g that some element of the row reaches: a vector whose largest
+// possible score, fma(max x, 1/T, kGumbelMax), stays below it cannot hold the
+// draw and skips its noise. Otherwise an element reaches the threshold only
+// if its noise exceeds t = thr - max x / T (less 0.01 for the rounding of the
+// noise and of the score), i.e. only if E = -log1p(-u) < exp(-t), i.e. only if
+// u < u_lim = -expm1(-exp(-t)). Since u_lim <= exp(-t), the words are cut at
+// the larger exp(-t + 0.001) (one ex2; the 0.001 covers its rounding): a word
+// above the cut has u > u_lim and skips both logarithms, and the elements let
+// through beyond u_lim score below the threshold, so the draw is the same.
+// Every element that reaches the test gets its exact score.
+template <int kN>
+__device__ __forceinline__ void gumbel_select(RowState& st, const float (&x)[kN], int v0,
+                                              const RowArgs& a, uint32_t row, float bound) {
   float vm = x[0];
 #pragma unroll
   for (int j = 1; j < kN; ++j) vm = fmaxf(vm, x[j]);
-  if (vm > st.m) {
-    if (kMode == kDraftArgmax) {
-      int jj = kN - 1;
-#pragma unroll
-      for (int j = kN - 1; j >= 0; --j)
-        if (x[j] == vm) jj = j;
-      st.bi = v0 + jj;
+  const float thr = fmaxf(bound, st.bz);
+  if (fmaf(vm, a.inv_t, kGumbelMax) < thr) return;
+  uint32_t w_cut = 0xffffffffu;
+  if (thr > -INFINITY) {
+    const float t = thr - vm * a.inv_t - 0.011f;
+    const float lim = ex2(-t * kLog2e);
+    // u(w) >= w 2^-32 (1 - 2^-23) for every word w, so u(w) <= lim only if
+    // w <= lim 2^32 (1 + 2^-22); the float product below rounds to no less.
+    if (lim < 1.f) {
+      const float c = lim * 0x1p32f * (1.f + 0x1p-21f);
+      w_cut = c >= 0x1p32f ? 0xffffffffu : static_cast<uint32_t>(c);
     }
-    absorb_max(st, vm, a.k2);
   }
-  if (st.m > -INFINITY) {
-    const float neg_mk = -st.m * a.k2;
-    float acc = 0.f;
+  // kN is 4 or 8 with v0 a multiple of 4: one Philox block per 4 elements.
 #pragma unroll
-    for (int j = 0; j < kN; ++j) acc += ex2(lg_term(x[j], a.k2, neg_mk));
-    st.s += acc;
-  }
-  if (kMode == kDraftGumbel) {
-    const float thr = fmaxf(bound, st.bz);
-    if (fmaf(vm, a.inv_t, kGumbelMax) < thr) return;
-    // An element of this vector reaches thr only if its noise exceeds
-    // t = thr - max x / T (less 0.01 for the rounding of the noise and of
-    // the score), i.e. only if E = -log1p(-u) < exp(-t), i.e. only if
-    // u < -expm1(-exp(-t)): larger u skip both logarithms.
-    float u_lim = 2.f;
-    if (thr > -INFINITY) {
-      const float t = thr - vm * a.inv_t - 0.01f;
-      u_lim = -expm1f(-expf(-t));
-    }
-    // kN is 4 or 8 with v0 a multiple of 4: one Philox block per 4 elements.
+  for (int q = 0; q < kN / 4; ++q) {
+    const uint32_t blk = static_cast<uint32_t>((v0 >> 2) + q);
+    const uint4 w = philox4x32_10(make_uint4(blk, row, a.ctr2, a.ctr3), a.key0, a.key1);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-    for (int q = 0; q < kN / 4; ++q) {
-      const uint32_t blk = static_cast<uint32_t>((v0 >> 2) + q);
-      const uint4 w = philox4x32_10(make_uint4(blk, row, a.ctr2, a.ctr3), a.key0, a.key1);
-      const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float u = uniform_from_word(ws[j]);
-        if (u > u_lim) continue;
-        const float z = fmaf(x[q * 4 + j], a.inv_t, gumbel_from_uniform(u));
-        const int v = v0 + q * 4 + j;
-        if (z > st.bz || (z == st.bz && v < st.bi)) {
-          st.bz = z;
-          st.bi = v;
-          st.bx = x[q * 4 + j];
-        }
+    for (int j = 0; j < 4; ++j) {
+      if (ws[j] > w_cut) continue;
+      const float z = fmaf(x[q * 4 + j], a.inv_t, gumbel_from_uniform(uniform_from_word(ws[j])));
+      const int v = v0 + q * 4 + j;
+      if (z > st.bz || (z == st.bz && v < st.bi)) {
+        st.bz = z;
+        st.bi = v;
+        st.bx = x[q * 4 + j];
       }
     }
   }
@@ -455,27 +444,22 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) row_pass_kernel(co
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[sidx]);
       const int e0 = (v_lo + c * kChunkVecs + tid) * kEpv;
+      float x[kVecsPerThread][kEpv];
+#pragma unroll
+      for (int k = 0; k < kVecsPerThread; ++k) widen<TIn>(v[k], x[k]);
+      absorb_chunk<kMode>(st, x, chunk_max<TIn>(v, x), e0, kConsumers * kEpv, a.k2);
       if (kMode == kDraftGumbel) {
         // The CTA's best score so far lets vectors that cannot win skip the
         // noise; each warp publishes its best after the stage.
         const float bound = order_float(*static_cast<volatile int*>(&best_score));
 #pragma unroll
-        for (int k = 0; k < kVecsPerThread; ++k) {
-          if (tid + k * kConsumers < nv) {
-            float x[kEpv];
-            widen<TIn>(v[k], x);
-            absorb<kMode>(st, x, e0 + k * kConsumers * kEpv, a, urow, bound);
-          }
-        }
+        for (int k = 0; k < kVecsPerThread; ++k)
+          if (tid + k * kConsumers < nv)
+            gumbel_select(st, x[k], e0 + k * kConsumers * kEpv, a, urow, bound);
         float wb = st.bz;
 #pragma unroll
         for (int d = 16; d >= 1; d >>= 1) wb = fmaxf(wb, __shfl_xor_sync(0xffffffffu, wb, d));
         if (lane == 0 && wb > bound) atomicMax(&best_score, float_order(wb));
-      } else {
-        float x[kVecsPerThread][kEpv];
-#pragma unroll
-        for (int k = 0; k < kVecsPerThread; ++k) widen<TIn>(v[k], x[k]);
-        absorb_chunk<kMode>(st, x, chunk_max<TIn>(v, x), e0, kConsumers * kEpv, a.k2);
       }
     }
     // Ragged tail: V % kEpv elements, on the last rank.
