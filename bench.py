@@ -104,6 +104,34 @@ def read_peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
 
 
+# ALU roofline of the draw at T > 0, bound by Philox4x32-10: 10 rounds per 4
+# words (one word per logit), each round two 32 x 32 -> 64-bit products, i.e.
+# four 32-bit multiply results: 10 integer multiply results per logit. Peak:
+# 64 such results per clock per SM (the CUDA programming guide's throughput
+# for compute capabilities 7.0 to 9.0, taken as unchanged) x SMs x max clock.
+PHILOX_MULS_PER_LOGIT = 10
+INT_MUL_PER_CLK_PER_SM = 64
+
+
+def alu_roofline(n_logits, ms, dev, kernel):
+    import torch
+
+    props = torch.cuda.get_device_properties(dev)
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            mhz = float(json.load(f)["sm_max_mhz"])
+    except Exception:
+        mhz = 2070.0
+    peak = INT_MUL_PER_CLK_PER_SM * props.multi_processor_count * mhz * 1e6 / 1e9
+    achieved = n_logits * PHILOX_MULS_PER_LOGIT / (ms * 1e-3) / 1e9
+    return {"bound": "alu", "achieved": round(achieved, 1), "peak": round(peak, 1),
+            "unit": "G int32 mul/s", "frac": round(achieved / peak, 4), "traffic": None,
+            "kernel": kernel, "algorithmic_muls": n_logits * PHILOX_MULS_PER_LOGIT,
+            "peak_source": (f"{INT_MUL_PER_CLK_PER_SM} 32-bit integer multiply results per clock "
+                            f"per SM x {props.multi_processor_count} SMs x {mhz:.0f} MHz "
+                            "(Philox4x32-10: 10 multiply results per logit)")}
+
+
 def roofline_entry(counts, attn_gbs, attn_tflops, hbm_peak, tf_peak, peak_src, traffic):
     """The attention kernel against the roofline that bounds it: HBM when its
     arithmetic intensity (algorithmic flops per algorithmic byte) is below the
@@ -694,7 +722,7 @@ def run_select(args):
             "launch": f"CUDA graphs of {n_rot} steps (programmatic dependent launch)",
         },
         "roofline": {
-            "bound": "hbm" if T == 0 else "alu",
+            "bound": "hbm",
             "achieved": round(draft_gbs, 1),
             "peak": hbm_peak,
             "unit": "GB/s",
@@ -703,7 +731,8 @@ def run_select(args):
             "kernel": "zarya_draft_select (row pass + selection), per call",
             "algorithmic_bytes": draft_bytes,
             "peak_source": f"{peak_src} HBM copy bandwidth",
-        },
+        } if T == 0 else alu_roofline(w.rows * w.V, draft_ms, dev,
+                                      "zarya_draft_select (row pass + selection), per call"),
         "e2e": {
             "value": round(replica_throughput(K, world, e2e_ms), 2),
             "unit": "steps/s",
@@ -947,10 +976,12 @@ def run_mode_a(args):
                    "plan_ms": round(plan_ms, 5),
                    "plan_steps_mean": float(n_steps.mean()),
                    "l2": f"{n_rot} rotating logits copies (> L2 between reuses)"},
-        "roofline": {"bound": "hbm" if temp == 0 else "alu", "achieved": round(gbs, 1),
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1),
                      "peak": hbm_peak, "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
                      "traffic": None, "kernel": "row_pass_kernel (zarya_sample_rows)",
-                     "algorithmic_bytes": nbytes, "peak_source": f"{peak_src} HBM copy bandwidth"},
+                     "algorithmic_bytes": nbytes, "peak_source": f"{peak_src} HBM copy bandwidth"}
+        if temp == 0 else alu_roofline(rows * w.V, step_ms, dev,
+                                       "row_pass_kernel (zarya_sample_rows)"),
         "e2e": None,
         "gpu_launches": K,
     }
