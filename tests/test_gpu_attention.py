@@ -69,9 +69,9 @@ def test_reduced_workload_matches_oracle_everywhere(zs, oracle_mod, name, mode):
                                        ("ragged_mid", None)])
 @pytest.mark.parametrize("splits", [1, 2, 3, 7])
 def test_split_kv_merge_matches_oracle(zs, oracle_mod, name, mode, splits):
-    """Forcing the key range to be split n ways (up to 8 splits form a
-    thread-block cluster and merge through distributed shared memory) still
-    matches the oracle."""
+    """Forcing the key range to be split n ways (up to 3 splits form a
+    thread-block cluster and merge through distributed shared memory, more
+    merge through the workspace) still matches the oracle."""
     w = wl.make(name, small=True)
     db = _run(zs, w, mode, kv_splits=splits)
     kc, vc = oracle_staged(oracle_mod, w)

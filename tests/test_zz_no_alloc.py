@@ -36,8 +36,8 @@ def _noalloc(zb, db, out):
                          db.slot_len, db.mask_mode, out, db.desc)
 
 
-# More than 8 key splits per tile merge through scratch memory (up to 8
-# merge inside a thread-block cluster); these plans need 9.5 to 14.5 MiB.
+# More than 3 key splits per tile merge through scratch memory (up to 3
+# merge inside a thread-block cluster); these plans need 8.6 to 12.1 MiB.
 @pytest.mark.parametrize("name,small,splits,override", [("decode_small", False, 9, {"B": 2}),
                                                         ("decode_small", False, 17, {"B": 1}),
                                                         ("decode_small", False, 12, {"B": 2})])
