@@ -429,9 +429,11 @@ zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int
  * node costs next to kernels. Not a step of the paper's method.
  *  src, dst: 16-byte aligned, ranges not overlapping; bytes: any (0 launches
  *            nothing). Ordered on `stream` like any kernel.
+ * The device is the stream's (or, while capturing or on the legacy stream,
+ * that of the device buffer); device memory must belong to it.
  * Returns ZARYA_ERR_INVALID_ARG (nothing launched) for a NULL or unaligned
- * pointer, memory the device cannot address, two host buffers, or
- * overlapping ranges.
+ * pointer, memory the device cannot address (another device's memory,
+ * pageable host memory), two host buffers, or overlapping ranges.
  */
 zarya_status zarya_copy(const void* src, void* dst, size_t bytes, zarya_stream_t stream);
 

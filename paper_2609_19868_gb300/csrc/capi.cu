@@ -620,16 +620,24 @@ zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the restore kernel", ce);
 }
 
-// The device address of `p` (device memory as is; page-locked host memory
-// through its mapping), or nullptr when the device cannot address it.
-static const void* device_address(const void* p, bool* is_device) {
-  cudaPointerAttributes a{};
-  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+// Pointer attributes, or false (the runtime's error cleared) for a pointer the
+// runtime cannot describe.
+static bool pointer_kind(const void* p, cudaPointerAttributes* a) {
+  *a = cudaPointerAttributes{};
+  if (cudaPointerGetAttributes(a, p) != cudaSuccess) {
     cudaGetLastError();   // clear the error the query leaves behind
-    return nullptr;
+    return false;
   }
-  *is_device = a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
-  if (*is_device) return p;
+  return true;
+}
+
+// The address through which the current device reaches `p`: device memory of
+// that device (or managed memory) as is, page-locked host memory through its
+// mapping; nullptr for anything else (another device's memory, pageable host
+// memory).
+static const void* device_address(const void* p, const cudaPointerAttributes& a, int dev) {
+  if (a.type == cudaMemoryTypeManaged) return p;
+  if (a.type == cudaMemoryTypeDevice) return a.device == dev ? p : nullptr;
   if (a.type != cudaMemoryTypeHost) return nullptr;
   void* d = nullptr;
   if (cudaHostGetDevicePointer(&d, const_cast<void*>(p), 0) != cudaSuccess) {
@@ -644,15 +652,23 @@ zarya_status zarya_copy(const void* src, void* dst, size_t bytes, zarya_stream_t
   if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u)
     return ZARYA_ERR_INVALID_ARG;
   if (bytes == 0) return ZARYA_OK;
-  bool src_dev = false, dst_dev = false;
-  const void* s = device_address(src, &src_dev);
-  const void* d = device_address(dst, &dst_dev);
-  if (s == nullptr || d == nullptr || (!src_dev && !dst_dev)) return ZARYA_ERR_INVALID_ARG;
-  const uintptr_t a = reinterpret_cast<uintptr_t>(s), b = reinterpret_cast<uintptr_t>(d);
-  if (a < b + bytes && b < a + bytes) return ZARYA_ERR_INVALID_ARG;   // overlapping ranges
+  cudaPointerAttributes as, ad;
+  if (!pointer_kind(src, &as) || !pointer_kind(dst, &ad)) return ZARYA_ERR_INVALID_ARG;
+  const auto on_device = [](const cudaPointerAttributes& a) {
+    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+  };
+  if (!on_device(as) && !on_device(ad)) return ZARYA_ERR_INVALID_ARG;   // two host buffers
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  cudaError_t ce = select_device(stream, src_dev ? src : dst);
+  cudaError_t ce = select_device(stream, on_device(as) ? src : dst);
   if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int dev = -1;
+  if ((ce = cudaGetDevice(&dev)) != cudaSuccess) return cuda_fail("cudaGetDevice", ce);
+  const void* s = device_address(src, as, dev);
+  const void* d = device_address(dst, ad, dev);
+  if (s == nullptr || d == nullptr) return ZARYA_ERR_INVALID_ARG;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(s), b = reinterpret_cast<uintptr_t>(d);
+  if ((a | b) & 15u) return ZARYA_ERR_INVALID_ARG;
+  if (a < b + bytes && b < a + bytes) return ZARYA_ERR_INVALID_ARG;   // overlapping ranges
   ce = launch_copy(s, const_cast<void*>(d), bytes, stream);
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the copy kernel", ce);
 }
