@@ -113,6 +113,18 @@ PHILOX_MULS_PER_LOGIT = 10
 INT_MUL_PER_CLK_PER_SM = 64
 
 
+def alu_roofline_entry(n_logits, ms, sms, mhz, kernel):
+    """The T > 0 draw against the integer-multiply peak of `sms` SMs at `mhz`."""
+    peak = INT_MUL_PER_CLK_PER_SM * sms * mhz * 1e6 / 1e9
+    achieved = n_logits * PHILOX_MULS_PER_LOGIT / (ms * 1e-3) / 1e9
+    return {"bound": "alu", "achieved": round(achieved, 1), "peak": round(peak, 1),
+            "unit": "G int32 mul/s", "frac": round(achieved / peak, 4), "traffic": None,
+            "kernel": kernel, "algorithmic_muls": n_logits * PHILOX_MULS_PER_LOGIT,
+            "peak_source": (f"{INT_MUL_PER_CLK_PER_SM} 32-bit integer multiply results per clock "
+                            f"per SM x {sms} SMs x {mhz:.0f} MHz "
+                            "(Philox4x32-10: 10 multiply results per logit)")}
+
+
 def alu_roofline(n_logits, ms, dev, kernel):
     import torch
 
@@ -122,14 +134,7 @@ def alu_roofline(n_logits, ms, dev, kernel):
             mhz = float(json.load(f)["sm_max_mhz"])
     except Exception:
         mhz = 2070.0
-    peak = INT_MUL_PER_CLK_PER_SM * props.multi_processor_count * mhz * 1e6 / 1e9
-    achieved = n_logits * PHILOX_MULS_PER_LOGIT / (ms * 1e-3) / 1e9
-    return {"bound": "alu", "achieved": round(achieved, 1), "peak": round(peak, 1),
-            "unit": "G int32 mul/s", "frac": round(achieved / peak, 4), "traffic": None,
-            "kernel": kernel, "algorithmic_muls": n_logits * PHILOX_MULS_PER_LOGIT,
-            "peak_source": (f"{INT_MUL_PER_CLK_PER_SM} 32-bit integer multiply results per clock "
-                            f"per SM x {props.multi_processor_count} SMs x {mhz:.0f} MHz "
-                            "(Philox4x32-10: 10 multiply results per logit)")}
+    return alu_roofline_entry(n_logits, ms, props.multi_processor_count, mhz, kernel)
 
 
 def roofline_entry(counts, attn_gbs, attn_tflops, hbm_peak, tf_peak, peak_src, traffic):
