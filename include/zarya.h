@@ -418,6 +418,33 @@ zarya_status zarya_restore(const int32_t* tokens, const int32_t* perm, const int
                            zarya_stream_t stream);
 
 /*
+ * Repetition penalty (Sec. 5.1 step 3 and Table 2: the per-step draws honour
+ * temperature, top_p and repetition_penalty; the paper names the parameter,
+ * and the reading here is the usual one for a generate() call): in place, for
+ * every row g of sequence b (rows desc->row_offsets[b] .. [b + 1] - 1) and
+ * every distinct token v among hist_tokens[hist_offsets[b] ..
+ * hist_offsets[b + 1] - 1], the logit x = logits[g, v] becomes x * penalty
+ * when x < 0 and x / penalty otherwise, computed in float32 (bf16 logits are
+ * rounded back to nearest even). A token that occurs several times is
+ * penalised once. Run it on the logits before zarya_draft_select,
+ * zarya_verify_accept or zarya_sample_rows.
+ *  logits       [desc->total_rows, desc->row_stride] of desc->dtype (read and
+ *               written; 16-byte aligned); rows of no sequence are untouched
+ *  hist_offsets [desc->batch + 1] int32, non-decreasing, last <= n_hist
+ *  hist_tokens  [n_hist] int32 (may be NULL when n_hist is 0)
+ *  penalty      > 0 and finite (1 changes nothing)
+ * desc supplies batch, vocab, dtype, total_rows, row_stride and row_offsets;
+ * its other fields are checked as for zarya_draft_select but not used.
+ * Device checks: a history range outside [0, n_hist] sets ZARYA_DEVERR_ROWS
+ * and leaves that row alone; a token outside [0, vocab) sets
+ * ZARYA_DEVERR_TOKEN and is skipped. Vocabularies above 1.6 M tokens return
+ * ZARYA_ERR_UNSUPPORTED.
+ */
+zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
+                                      const int32_t* hist_tokens, int32_t n_hist, float penalty,
+                                      const zarya_sample_desc* desc, zarya_stream_t stream);
+
+/*
  * Moves `bytes` bytes from src to dst with a kernel instead of a copy engine:
  * a grid of at most 24 CTAs reads and writes 16-byte vectors, reaching host
  * memory through its device mapping. Each of src and dst is device memory or

@@ -116,6 +116,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_draft_select.restype = ctypes.c_int
     lib.zarya_verify_accept.argtypes = [vp] * 7 + [sp, vp]
     lib.zarya_verify_accept.restype = ctypes.c_int
+    lib.zarya_repetition_penalty.argtypes = [vp, vp, vp, i32, ctypes.c_float, sp, vp]
+    lib.zarya_repetition_penalty.restype = ctypes.c_int
     lib.zarya_copy.argtypes = [vp, vp, sz, vp]
     lib.zarya_copy.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
@@ -318,6 +320,21 @@ def sample_rows(logits, tokens, prob, desc: SampleDesc, stream=None) -> None:
                                   _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_sample_rows")
+
+
+def repetition_penalty(logits, hist_offsets, hist_tokens, penalty: float, desc: SampleDesc,
+                       stream=None) -> None:
+    """``zarya_repetition_penalty``: in place, the logits of every token in a
+    row's sequence history multiplied by ``penalty`` when negative, divided by
+    it otherwise (Sec. 5.1 step 3, Table 2)."""
+    _check_logits(logits, desc)
+    _check_cuda("hist_offsets", hist_offsets, torch.int32)
+    _check_cuda("hist_tokens", hist_tokens, torch.int32)
+    st = load().zarya_repetition_penalty(_ptr(logits), _ptr(hist_offsets), _ptr(hist_tokens),
+                                         hist_tokens.numel(), float(penalty), ctypes.byref(desc),
+                                         _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_repetition_penalty")
 
 
 def mode_a_budget(n_masked, T: int, alpha0: float, seed: int, offset: int, counts, n_steps,

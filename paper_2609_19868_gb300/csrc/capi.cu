@@ -542,6 +542,37 @@ zarya_status zarya_sample_rows(const void* logits, int32_t* tokens, float* prob,
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the row-sampling kernel", ce);
 }
 
+zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
+                                      const int32_t* hist_tokens, int32_t n_hist, float penalty,
+                                      const zarya_sample_desc* desc, zarya_stream_t stream_) {
+  zarya_status st = check_sample_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!logits || !hist_offsets || !aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
+  if (n_hist < 0 || (n_hist > 0 && !hist_tokens)) return ZARYA_ERR_INVALID_ARG;
+  if (!(penalty > 0.f) || std::isinf(penalty)) return ZARYA_ERR_INVALID_ARG;
+  if (static_cast<size_t>((desc->vocab + 31) / 32) * 4 > 200 * 1024) return ZARYA_ERR_UNSUPPORTED;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, logits);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  int* err = device_error_word(&ce);
+  if (err == nullptr) return cuda_fail("looking up the device error word", ce);
+  PenaltyParams p{};
+  p.logits = logits;
+  p.row_offsets = desc->row_offsets;
+  p.hist_offsets = hist_offsets;
+  p.hist_tokens = hist_tokens;
+  p.err = err;
+  p.B = desc->batch;
+  p.V = desc->vocab;
+  p.rows = desc->total_rows;
+  p.n_hist = n_hist;
+  p.row_stride = desc->row_stride;
+  p.penalty = penalty;
+  p.bf16 = desc->dtype == ZARYA_BF16 ? 1 : 0;
+  ce = launch_penalty(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the repetition-penalty kernel", ce);
+}
+
 zarya_status zarya_mode_a_budget(const int32_t* n_masked, int32_t batch, int32_t T, float alpha0,
                                  uint64_t seed, uint64_t offset, int32_t max_steps,
                                  int32_t* counts, int32_t* n_steps, zarya_stream_t stream_) {

@@ -18,6 +18,21 @@ cudaError_t launch_sample_rows(const SampleCall& c, int32_t* tokens, float* prob
 // device mapping of page-locked host memory); src and dst 16-byte aligned.
 cudaError_t launch_copy(const void* src, void* dst, size_t bytes, cudaStream_t stream);
 
+// Repetition penalty over logits rows, in place.
+struct PenaltyParams {
+  void* logits;                // [rows, row_stride] bf16 or fp32
+  const int32_t* row_offsets;  // [B + 1] rows of each sequence
+  const int32_t* hist_offsets; // [B + 1] history tokens of each sequence
+  const int32_t* hist_tokens;  // [n_hist]
+  int* err;
+  int B, V, rows, n_hist;
+  int64_t row_stride;          // elements
+  float penalty;
+  int bf16;
+};
+
+cudaError_t launch_penalty(const PenaltyParams& p, cudaStream_t stream);
+
 // Reordering / restoration of [B, max_len] token rows.
 struct ReorderParams {
   const int32_t* tokens;

@@ -290,3 +290,23 @@ def test_copy_binding_checks_tensors():
     a = torch.zeros(16, dtype=torch.uint8)
     with pytest.raises(TypeError):
         zb.copy(a, a.clone())       # neither pinned nor on a device
+
+
+def test_repetition_penalty_rejects_invalid_calls(lib):
+    vp = ctypes.c_void_p
+
+    def call(logits=FAKE, offs=FAKE + 64, toks=FAKE + 128, n=4, p=1.2, d="ok"):
+        desc = _sdesc() if d == "ok" else d
+        return lib.zarya_repetition_penalty(vp(logits), vp(offs), vp(toks), n, p,
+                                            None if desc is None else ctypes.byref(desc), None)
+
+    assert call(logits=None) == 1
+    assert call(logits=FAKE + 8) == 1           # unaligned logits
+    assert call(offs=None) == 1
+    assert call(toks=None) == 1                 # tokens promised but missing
+    assert call(n=-1) == 1
+    for p in (0.0, -1.0, float("nan"), float("inf")):
+        assert call(p=p) == 1
+    assert call(d=None) == 1
+    assert call(d=_sdesc(vocab=0)) == 1
+    assert call(d=_sdesc(vocab=2_000_000, row_stride=2_000_000)) == 2   # bitmap too large
