@@ -445,6 +445,31 @@ zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
                                       const zarya_sample_desc* desc, zarya_stream_t stream);
 
 /*
+ * top_p (nucleus) truncation (Sec. 5.1 step 3 and Table 2; the paper names
+ * the parameter, and the reading here is nucleus sampling): in place, for
+ * every row of a sequence (rows desc->row_offsets[0] .. [batch] - 1), with
+ * p = softmax(x / T) (softmax(x) when desc->temperature is 0), the logits
+ * below x* become -inf, where x* is the largest logit value such that the
+ * tokens at or above it hold at least top_p of the row's probability: the
+ * smallest set of most probable tokens reaching top_p, with every token tied
+ * at its boundary kept. A draw that follows (zarya_draft_select,
+ * zarya_verify_accept, zarya_sample_rows with the same temperature) then runs
+ * over the nucleus, each token with its usual noise, and reports
+ * probabilities renormalised over it. The masses behind the boundary are
+ * summed in 2^-40 fixed point, so the result does not depend on the order of
+ * the GPU's additions; it can differ from exact arithmetic only where the
+ * mass at a boundary lies within about 1e-6 of top_p.
+ *  logits   [desc->total_rows, desc->row_stride] of desc->dtype (read and
+ *           written; 16-byte aligned); rows of no sequence are untouched
+ *  top_p    in (0, 1); top_p >= 1 returns at once (nothing to cut)
+ * desc supplies batch, vocab, dtype, total_rows, row_stride, row_offsets and
+ * temperature; its other fields are checked as for zarya_draft_select.
+ * Returns ZARYA_ERR_INVALID_ARG for top_p <= 0 or NaN.
+ */
+zarya_status zarya_top_p(void* logits, float top_p, const zarya_sample_desc* desc,
+                         zarya_stream_t stream);
+
+/*
  * Moves `bytes` bytes from src to dst with a kernel instead of a copy engine:
  * a grid of at most 24 CTAs reads and writes 16-byte vectors, reaching host
  * memory through its device mapping. Each of src and dst is device memory or

@@ -118,6 +118,8 @@ def load() -> ctypes.CDLL:
     lib.zarya_verify_accept.restype = ctypes.c_int
     lib.zarya_repetition_penalty.argtypes = [vp, vp, vp, i32, ctypes.c_float, sp, vp]
     lib.zarya_repetition_penalty.restype = ctypes.c_int
+    lib.zarya_top_p.argtypes = [vp, ctypes.c_float, sp, vp]
+    lib.zarya_top_p.restype = ctypes.c_int
     lib.zarya_copy.argtypes = [vp, vp, sz, vp]
     lib.zarya_copy.restype = ctypes.c_int
     lib.zarya_check_device_error.argtypes = [vp, ctypes.POINTER(i32)]
@@ -335,6 +337,16 @@ def repetition_penalty(logits, hist_offsets, hist_tokens, penalty: float, desc: 
                                          _stream(stream))
     if st != OK:
         raise ZaryaError(st, "zarya_repetition_penalty")
+
+
+def top_p(logits, top_p: float, desc: SampleDesc, stream=None) -> None:
+    """``zarya_top_p``: in place, the logits outside each row's nucleus (the
+    smallest most-probable set reaching ``top_p`` under softmax(x / T))
+    become -inf (Sec. 5.1 step 3, Table 2)."""
+    _check_logits(logits, desc)
+    st = load().zarya_top_p(_ptr(logits), float(top_p), ctypes.byref(desc), _stream(stream))
+    if st != OK:
+        raise ZaryaError(st, "zarya_top_p")
 
 
 def mode_a_budget(n_masked, T: int, alpha0: float, seed: int, offset: int, counts, n_steps,

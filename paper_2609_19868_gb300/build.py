@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libzarya.so")
 SOURCES = ["capi.cu", "slot_attn_tc.cu", "simt_kernels.cu", "noalloc.cu", "sampling.cu", "reorder.cu",
-           "mode_a.cu", "copy.cu", "penalty.cu"]
+           "mode_a.cu", "copy.cu", "penalty.cu", "nucleus.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

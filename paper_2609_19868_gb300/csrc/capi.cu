@@ -573,6 +573,30 @@ zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
   return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the repetition-penalty kernel", ce);
 }
 
+zarya_status zarya_top_p(void* logits, float top_p, const zarya_sample_desc* desc,
+                         zarya_stream_t stream_) {
+  zarya_status st = check_sample_desc(desc);
+  if (st != ZARYA_OK) return st;
+  if (!logits || !aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
+  if (!(top_p > 0.f)) return ZARYA_ERR_INVALID_ARG;   // also NaN
+  if (top_p >= 1.f) return ZARYA_OK;                  // the nucleus is the whole vocabulary
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t ce = select_device(stream, logits);
+  if (ce != cudaSuccess) return cuda_fail("selecting the stream's device", ce);
+  NucleusParams p{};
+  p.logits = logits;
+  p.row_offsets = desc->row_offsets;
+  p.B = desc->batch;
+  p.V = desc->vocab;
+  p.rows = desc->total_rows;
+  p.row_stride = desc->row_stride;
+  p.k2 = desc->temperature > 0.f ? 1.4426950408889634f / desc->temperature : 1.4426950408889634f;
+  p.top_p = top_p;
+  p.bf16 = desc->dtype == ZARYA_BF16 ? 1 : 0;
+  ce = launch_nucleus(p, stream);
+  return ce == cudaSuccess ? ZARYA_OK : cuda_fail("launching the top_p kernel", ce);
+}
+
 zarya_status zarya_mode_a_budget(const int32_t* n_masked, int32_t batch, int32_t T, float alpha0,
                                  uint64_t seed, uint64_t offset, int32_t max_steps,
                                  int32_t* counts, int32_t* n_steps, zarya_stream_t stream_) {

@@ -33,6 +33,19 @@ struct PenaltyParams {
 
 cudaError_t launch_penalty(const PenaltyParams& p, cudaStream_t stream);
 
+// top_p truncation of logits rows, in place.
+struct NucleusParams {
+  void* logits;                // [rows, row_stride] bf16 or fp32
+  const int32_t* row_offsets;  // [B + 1] rows of each sequence
+  int B, V, rows;
+  int64_t row_stride;          // elements
+  float k2;                    // log2(e) / T (log2(e) at T = 0)
+  float top_p;
+  int bf16;
+};
+
+cudaError_t launch_nucleus(const NucleusParams& p, cudaStream_t stream);
+
 // Reordering / restoration of [B, max_len] token rows.
 struct ReorderParams {
   const int32_t* tokens;

@@ -310,3 +310,14 @@ def test_repetition_penalty_rejects_invalid_calls(lib):
     assert call(d=None) == 1
     assert call(d=_sdesc(vocab=0)) == 1
     assert call(d=_sdesc(vocab=2_000_000, row_stride=2_000_000)) == 2   # bitmap too large
+
+
+def test_top_p_rejects_invalid_calls(lib):
+    vp = ctypes.c_void_p
+    d = _sdesc()
+    assert lib.zarya_top_p(vp(None), 0.9, ctypes.byref(d), None) == 1
+    assert lib.zarya_top_p(vp(FAKE + 8), 0.9, ctypes.byref(d), None) == 1
+    for p in (0.0, -0.5, float("nan")):
+        assert lib.zarya_top_p(vp(FAKE), p, ctypes.byref(d), None) == 1
+    assert lib.zarya_top_p(vp(FAKE), 0.9, None, None) == 1
+    assert lib.zarya_top_p(vp(FAKE), 1.0, ctypes.byref(d), None) == 0   # nothing to cut

@@ -1,0 +1,122 @@
+"""zarya_top_p against the oracle (oracle/nucleus.py): the kept set of every
+row on fp32 and bf16 rows (heavy ties in bf16), several temperatures and top_p
+values, rows of no sequence, and draws taken after the truncation. The GPU
+sums masses in fixed point from fp32 exponentials, so a kept set may differ
+from the exact one only where the mass at a boundary is within 1e-5 of
+top_p; every difference is checked to be such a case."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import nucleus as nuc
+from oracle import penalty as pen
+from oracle import sampling as smp
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def zb():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_19868_gb300 import build
+    from paper_2609_19868_gb300 import _binding as zb
+
+    build.build()
+    zb.load()
+    zb.check_device_error()
+    return zb
+
+
+def _i32(a):
+    return torch.as_tensor(np.asarray(a, dtype=np.int32)).cuda()
+
+
+def _run(zb, x, dtype, row_offsets, T, top_p, max_slots=1):
+    rows, V = x.shape
+    epv = 8 if dtype == torch.bfloat16 else 4
+    stride = (V + epv - 1) // epv * epv
+    buf = torch.full((rows, stride), float("nan"), dtype=dtype, device="cuda")
+    buf[:, :V] = torch.as_tensor(x).to(dtype).cuda()
+    logits = buf.as_strided((rows, V), (stride, 1))
+    ro = _i32(row_offsets)
+    d = zb.make_sample_desc(batch=len(row_offsets) - 1, vocab=V,
+                            dtype=zb.BF16 if dtype == torch.bfloat16 else zb.FP32,
+                            max_slots=max_slots, total_rows=rows, row_stride=stride,
+                            temperature=T, slot_threshold=0.9, token_threshold=0.4, seed=7,
+                            offset=1, row_offsets=ro)
+    zb.top_p(logits, top_p, d)
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    return logits, ro, d
+
+
+def _kept_ok(x_row, gpu_kept, T, top_p):
+    """The GPU's kept set (over the finite logits) equals the oracle's, or
+    differs only at boundaries whose exact mass is within 1e-5 of top_p."""
+    fin = np.isfinite(x_row)
+    want = nuc.kept_mask(x_row, T, top_p)
+    if np.array_equal(gpu_kept[fin], want[fin]):
+        return True
+    p = nuc._probs(x_row, T)
+    for v in np.unique(x_row[fin & (gpu_kept != want)]):
+        if min(abs(p[x_row >= v].sum() - top_p), abs(p[x_row > v].sum() - top_p)) > 1e-5:
+            return False
+    return True
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("V", [37, 4099, 151936])
+def test_kept_sets_match_the_oracle(zb, dtype, V):
+    rng = np.random.default_rng(V)
+    grid = [(T, p) for T in (0.0, 0.6, 1.0, 1.9) for p in (0.05, 0.5, 0.9, 0.99)]
+    if V > 100000:   # the oracle walks up to the whole row in Python: a few cases suffice
+        grid = [(0.0, 0.5), (1.0, 0.99), (0.6, 0.05)]
+    for T, top_p in grid:
+        rows = 5
+        scale = float(rng.choice([0.5, 2.0, 4.0]))
+        x = rng.normal(scale=scale, size=(rows, V)).astype(np.float32)
+        x[0, : V // 3] = -np.inf                      # a row with tokens already cut
+        if dtype == torch.bfloat16:
+            x = np.where(np.isfinite(x), pen.bf16_round(np.where(np.isfinite(x), x, 0.0)), x)
+        ro = [0, 2, 4]                                # row 4 belongs to no sequence
+        logits, _, _ = _run(zb, x, dtype, ro, T, top_p)
+        got = logits.float().cpu().numpy()
+        for g in range(4):
+            kept = np.isfinite(got[g])
+            assert np.array_equal(got[g][kept], x[g][kept])      # kept logits unchanged
+            assert (got[g][~kept] == -np.inf).all()               # the rest cut
+            assert kept.any()
+            assert _kept_ok(x[g].astype(np.float64), kept, T, top_p), (T, top_p, g)
+        assert np.array_equal(got[4], x[4])           # a row of no sequence: untouched
+
+
+@pytest.mark.parametrize("T", [0.0, 0.8])
+def test_draws_after_top_p_stay_in_the_nucleus(zb, T):
+    rng = np.random.default_rng(11)
+    B, S, L, V = 2, 2, 4, 2053
+    rows = B * S * L
+    x = rng.normal(scale=2.0, size=(rows, V)).astype(np.float32)
+    ro = np.arange(0, rows + 1, S * L, dtype=np.int32)
+    logits, ro_dev, d = _run(zb, x, torch.float32, ro, T, 0.6, max_slots=S)
+    kept_gpu = np.isfinite(logits.float().cpu().numpy())
+    dev_i32 = lambda n, v: torch.full((n,), v, dtype=torch.int32, device="cuda")  # noqa: E731
+    tok = dev_i32(rows, -7)
+    prob = torch.full((rows,), -7.0, device="cuda")
+    zb.draft_select(logits, dev_i32(B, S), dev_i32(B, L), tok, prob,
+                    torch.zeros((B, S), device="cuda"),
+                    torch.zeros((B, S), dtype=torch.uint8, device="cuda"), dev_i32(B, -7),
+                    dev_i32(B + 1, -7), dev_i32(rows, -7), dev_i32(rows, -7), d)
+    torch.cuda.synchronize()
+    assert zb.check_device_error() == 0
+    tok, prob = tok.cpu().numpy(), prob.cpu().numpy()
+    g_noise = lambda g: smp.gumbel_noise(7, 1, g, V)      # noqa: E731
+    for g in range(rows):
+        xg = x[g].astype(np.float64)
+        assert kept_gpu[g][tok[g]]                                      # inside the nucleus
+        want = nuc.draw_token(xg, T, 0.6, 7, 1, g)
+        if tok[g] != want:   # only a near-tie of two kept scores may differ
+            z = xg / T + g_noise(g) if T > 0 else xg
+            assert abs(z[tok[g]] - z[want]) < 1e-4 * (1 + abs(z[want]))
+        p_ref = nuc.row_probability(xg, int(tok[g]), T, 0.6)
+        assert abs(prob[g] - p_ref) < 1e-5 + 1e-4 * p_ref
