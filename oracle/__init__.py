@@ -4,7 +4,7 @@ TEST INFRASTRUCTURE ONLY. Only ``tests/``, ``__graft_entry__.smoke()`` and
 the CPU-baseline leg of ``bench.py`` may import this package. It shares no
 code with the CUDA library and never imports it.
 
-Three independent formulations live here:
+The package holds these formulations, each written from the paper:
 
 * ``slot_attn`` / ``slot_attn_rows``: the C implementation in
   ``slot_attn_oracle.c`` (masked softmax attention written out by its
@@ -17,6 +17,12 @@ Three independent formulations live here:
 * ``oracle.sampling``: slot selection and token acceptance (Sec. 5.2 steps
   3-6): draws, Gumbel-max sampling, slot confidences, the selection rule and
   the accepted prefixes, in numpy fp64.
+* ``oracle.mode_a``: Mode A's mask-budget plan and per-step draws (Sec. 5.1
+  steps 1 and 3).
+* ``oracle.reorder``: reordering and restoration (Sec. 5.1 steps 2 and 4,
+  Sec. 5.2 steps 1 and 8).
+* ``oracle.penalty`` and ``oracle.nucleus``: the repetition penalty and top_p
+  truncation the per-step draws honour (Sec. 5.1 step 3, Table 2).
 
 Mask modes (Sec. 5.2):
   0  block-bidirectional (draft pass, step 3): block rows see the whole prefix
