@@ -67,3 +67,17 @@ def test_renormalised_probabilities():
     assert nuc.row_probability(P4, 0, 1.0, 0.7) == pytest.approx(0.5 / 0.8, rel=1e-12)
     assert nuc.row_probability(P4, 2, 1.0, 0.7) == 0.0
     assert nuc.row_probability(P4, 3, 1.0, 1.0) == pytest.approx(0.05, rel=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_threshold_against_every_candidate_value(seed):
+    # x* is the largest logit value v whose tokens at or above it hold at least
+    # top_p of the mass: checked by trying every distinct value
+    rng = np.random.default_rng(seed)
+    x = np.round(rng.normal(scale=2, size=300), 1)      # many ties
+    for T in (0.0, 0.7):
+        p = nuc._probs(x, T)
+        for top_p in (0.1, 0.5, 0.8, 0.97):
+            vals = np.unique(x)[::-1]
+            ok = [v for v in vals if p[x >= v].sum() >= top_p]
+            assert nuc.kept_threshold(x, T, top_p) == max(ok)

@@ -101,3 +101,13 @@ def test_brute_force_definition(dtype):
                 assert out[g, v] == want, (b, g, v)
     assert np.array_equal(out[5], x[5])            # row 5 belongs to no sequence
     assert bad == bool(((hist < 0) | (hist >= V)).any())
+
+
+def test_bf16_rounding_agrees_with_torch_conversion():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(7)
+    x = np.concatenate([rng.normal(scale=s, size=4000) for s in (1e-3, 1.0, 1e3, 1e30)])
+    x = x.astype(np.float32)
+    ours = pen.bf16_round(x)
+    lib = torch.from_numpy(x).to(torch.bfloat16).float().numpy()
+    assert np.array_equal(ours.view(np.uint32), lib.view(np.uint32))
