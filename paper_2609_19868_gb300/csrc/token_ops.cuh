@@ -1,6 +1,7 @@
 // Declarations of the token-level kernels that sit around the attention
-// step (row sampling of Mode A, reordering / restoration, Mode A planning),
-// shared by their translation units and the C ABI.
+// step (row sampling of Mode A, the repetition penalty and top_p truncation
+// of logits, reordering / restoration, Mode A planning) and of the SM copy
+// kernel, shared by their translation units and the C ABI.
 #pragma once
 
 #include <cuda_runtime.h>
