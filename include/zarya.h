@@ -6,7 +6,12 @@
  * Autoregressive--Masked Diffusion Language Model with Flexible Training and
  * Dual-Mode Inference") and the KV-cache update with accepted tokens that
  * gives the mode its full KV reuse (Sec. 5.2 step 7; Sec. 5.1 explains why the
- * reordered prefix cache stays valid under causal attention).
+ * reordered prefix cache stays valid under causal attention). Around it sit
+ * the token-level steps of both inference modes: slot selection and token
+ * acceptance (Sec. 5.2 steps 3-6), Mode A's reveal plan and per-step draws
+ * (Sec. 5.1 steps 1 and 3) with the repetition penalty and top_p they honour
+ * (Table 2), and the reordering / restoration of sequences (Sec. 5.1 steps 2
+ * and 4, Sec. 5.2 steps 1 and 8).
  *
  * Notation: sequence b of a batch of B; committed prefix length
  * P_b = cache_lens[b]; the current block holds S_b = n_slots[b] slots of
@@ -19,8 +24,9 @@
  *
  * General rules for every entry point:
  *  - All array arguments are DEVICE pointers on the device that owns `stream`
- *    (the caller owns every buffer). Calls are asynchronous on `stream`; none
- *    blocks except zarya_check_device_error.
+ *    (the caller owns every buffer), except where a call says otherwise
+ *    (zarya_copy also takes page-locked host buffers). Calls are asynchronous
+ *    on `stream`; none blocks except zarya_check_device_error.
  *  - Host-side validation happens first; an invalid call returns a status and
  *    launches nothing. Nothing falls back to the CPU.
  *  - Errors that only the device can see (a page id out of range, a length
