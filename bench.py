@@ -8,10 +8,18 @@ One step = the whole hot path over one batch:
 The commit writes the advanced lengths into a second array (a decoding
 loop's ping-pong), so every step sees the same prefix lengths.
 
-Default workload: decode_small (B8, 16/8 heads, D128, bf16, P=2048,
-contiguous cache, 4 slots x 8 tokens, slot-causal). Inputs are seeded and
-synthetic. Several independent copies of the KV cache rotate so that the
-data touched between two uses of one copy exceeds the L2 cache.
+Default workload: serving_mix (B64, 32/8 heads, D128, bf16, paged cache of
+16-token pages, prefixes log-uniform in [1024, 16384], 8 slots of 4 to 32
+tokens, mask mode per sequence), the largest configuration. Inputs are
+seeded and synthetic. Several independent copies of the KV cache rotate so
+that the data touched between two uses of one copy exceeds the L2 cache.
+
+Every measurement is a series of timed regions of K steps (at least --reps
+of them, lasting at least --min-seconds), reported as the median region
+(the minimum beside it). The line's `per_config` object repeats the
+measurement for every configuration (tiny_fp32, decode_small, ragged_mid,
+long_ctx in both mask modes, serving_mix), each with its roofline, the
+oracle's time on the host cores and the end-to-end rate with host buffers.
 
 Prints one JSON line. `--impl reference` times the fp64 CPU oracle instead
 (rank 0 only), each step a bounded sample of the same workload.
@@ -41,15 +49,21 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 
 WORKLOAD_LABELS = {
+    "tiny_fp32": "tiny_fp32: B1, Hq4/Hkv2, D64, fp32, prefix 128, contiguous cache, "
+                 "2 slots x 4 tokens, slot-causal, accept 3",
     "decode_small": "decode_small: B8, Hq16/Hkv8, D128, bf16, prefix 2048, contiguous cache, "
                     "4 slots x 8 tokens, slot-causal, accept ~U[0,R]",
     "ragged_mid": "ragged_mid: B32, Hq32/Hkv8, D128, bf16, prefix ~U[512,8192], contiguous, "
                   "8 slots x 16 tokens, block-bidirectional",
-    "long_ctx": "long_ctx: B4, Hq32/Hkv8, D128, bf16, prefix 32768, contiguous, "
-                "16 slots x 32 tokens, slot-causal",
+    "long_ctx_bidir": "long_ctx: B4, Hq32/Hkv8, D128, bf16, prefix 32768, contiguous, "
+                      "16 slots x 32 tokens, block-bidirectional, accept ~U[0,512]",
+    "long_ctx_causal": "long_ctx: B4, Hq32/Hkv8, D128, bf16, prefix 32768, contiguous, "
+                       "16 slots x 32 tokens, slot-causal, accept ~U[0,512]",
     "serving_mix": "serving_mix: B64, Hq32/Hkv8, D128, bf16, paged 16-token pages, prefix "
                    "log-U[1024,16384], slot_len in {4,8,16,32} x 8 slots, mixed modes",
 }
+# older name of the slot-causal long_ctx entry
+WORKLOAD_ALIASES = {"long_ctx": "long_ctx_causal"}
 
 
 def algorithmic_counts(w):
@@ -182,7 +196,9 @@ class ClockSampler:
             self.proc = None
         return self
 
-    def stop(self, t0: float, t1: float):
+    def stop(self, t0: float, t1: float, keep: bool = False):
+        """Ends the sampling and returns the clocks seen in [t0, t1]; with
+        `keep`, the samples stay available to window()."""
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.proc.terminate()
@@ -203,6 +219,15 @@ class ClockSampler:
                     rows.append((ts + frac, float(parts[2]), float(parts[3]), parts[5:9]))
                 except Exception:
                     continue
+        self.rows = rows
+        return self.window(t0, t1)
+
+    def window(self, t0: float, t1: float):
+        """Median SM clock, maximum clock and throttle reasons of the samples
+        taken in [t0, t1] (the nearest sample when none falls inside)."""
+        rows = getattr(self, "rows", None)
+        if self.proc is None or rows is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         inside = [r for r in rows if t0 - 0.05 <= r[0] <= t1 + 0.05]
         used = inside
         note = None
@@ -214,7 +239,8 @@ class ClockSampler:
         reasons = sorted({names[i] for r in used for i, v in enumerate(r[3]) if v == "Active"})
         out = {"sm_mhz": float(np.median([r[1] for r in used])) if used else None,
                "sm_max_mhz": max(r[2] for r in used) if used else None,
-               "reasons": reasons, "samples": len(inside)}
+               "reasons": reasons, "samples": len(inside),
+               "window_s": round(t1 - t0, 3)}
         if note:
             out["note"] = note
         return out
@@ -246,45 +272,151 @@ def replica_throughput(steps: int, world: int, total_ms: float) -> float:
     return steps * world / (total_ms * 1e-3)
 
 
-def run_ours(args):
+def per_sequence_roofline(w, hbm_peak, tf_peak):
+    """Ideal time of the attention launch under a roofline taken sequence by
+    sequence: every sequence b needs at least max(bytes_b / HBM, flops_b /
+    bf16) (its K/V, Q and O bytes; 4 D flops per visible pair), and the batch
+    needs their sum. For a batch whose sequences all have the same shape this
+    is the usual single-intensity roofline. Returns (ideal_s, hbm_part_s,
+    tensor_part_s, batch_wide_s), the last being max(sum bytes / HBM,
+    sum flops / bf16), a lower bound on the same time."""
+    eb = 2 if w.dtype == "bf16" else 4
+    P = w.cache_lens.astype(np.int64)
+    R = w.R
+    kv = w.Hkv * (P + R) * w.D * eb * 2
+    qo = 2 * R * w.Hq * w.D * eb
+    pairs = np.where(w.mask_mode == 0, w.Hq * R * (P + R), w.Hq * (R * P + R * (R + 1) // 2))
+    byts = (kv + qo).astype(np.float64)
+    flops = (4 * w.D * pairs).astype(np.float64)
+    t_hbm = byts / (hbm_peak * 1e9)
+    t_tc = flops / (tf_peak * 1e12)
+    ideal = float(np.maximum(t_hbm, t_tc).sum())
+    hbm_part = float(np.where(t_hbm >= t_tc, t_hbm, 0.0).sum())
+    batch_wide = max(float(byts.sum()) / (hbm_peak * 1e9), float(flops.sum()) / (tf_peak * 1e12))
+    return ideal, hbm_part, ideal - hbm_part, batch_wide
+
+
+def roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src, traffic):
+    """The attention launch against the per-sequence roofline of its batch.
+
+    `bound` names the resource that bounds most of the ideal time. When every
+    sequence is bound by the same resource, `peak` is that resource's measured
+    peak and `achieved` the algorithmic bytes (HBM) or flops (tensor) per
+    second. When the batch mixes HBM-bound and tensor-bound sequences, the
+    bound is the dominant one and `peak` is the rate the roofline allows for
+    this batch (its algorithmic amount / the ideal time), so that
+    frac = achieved / peak = ideal time / measured time."""
+    ideal, hbm_part, tc_part, batch_wide = per_sequence_roofline(w, hbm_peak, tf_peak)
+    t = attn_ms * 1e-3
+    frac = ideal / t
+    if tc_part >= hbm_part:
+        bound, unit, amount, peak_meas = "tensor", "TFLOP/s", counts["flops"] / 1e12, tf_peak
+        src = f"{peak_src} cuBLAS bf16 GEMM (burst)"
+    else:
+        bound, unit, amount, peak_meas = "hbm", "GB/s", counts["attn_bytes"] / 1e9, hbm_peak
+        src = f"{peak_src} HBM copy bandwidth"
+    achieved = amount / t
+    mixed = hbm_part > 0 and tc_part > 0
+    peak = amount / ideal if mixed else peak_meas
+    entry = {"bound": bound, "achieved": round(achieved, 1), "peak": round(peak, 1), "unit": unit,
+             "frac": round(achieved / peak, 4), "traffic": traffic,
+             "peak_source": (f"per-sequence roofline of this batch (sum over sequences of "
+                             f"max(bytes_b / {hbm_peak:.0f} GB/s, flops_b / {tf_peak:.0f} TFLOP/s), "
+                             f"{peak_src} peaks): the attainable rate" if mixed else src),
+             "ideal_us": round(ideal * 1e6, 2),
+             "ideal_us_hbm_bound_sequences": round(hbm_part * 1e6, 2),
+             "ideal_us_tensor_bound_sequences": round(tc_part * 1e6, 2),
+             "frac_of_batch_wide_bound": round(batch_wide / t, 4),
+             "intensity_flop_per_byte": round(counts["flops"] / counts["attn_bytes"], 1),
+             "ridge_flop_per_byte": round(tf_peak * 1e12 / (hbm_peak * 1e9), 1),
+             "kernel": "slot_attn_tc_kernel" if w.dtype == "bf16" else "slot_attn_f32_kernel"}
+    if mixed:
+        entry["peak_measured"] = peak_meas
+    if w.dtype != "bf16":
+        entry["note"] = ("fp32 correctness configuration on the CUDA cores: a few microseconds "
+                         "of launch latency, far from any throughput roof")
+    return entry
+
+
+def timed_reps(enqueue, stream, min_reps, min_seconds, max_reps=20000):
+    """Times `enqueue()` (which enqueues one K-step region on `stream`) over
+    repeated regions: one calibration region, then n >= min_reps regions back
+    to back with a CUDA event between consecutive ones, n chosen so that the
+    whole run lasts at least min_seconds. Returns (per-region ms list,
+    wall-clock start, wall-clock end)."""
     import torch
-    import torch.distributed as dist
 
-    world, rank, local = dist_setup()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-    from paper_2609_19868_gb300 import build as zbuild
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0.record(stream)
+    enqueue()
+    c1.record(stream)
+    torch.cuda.synchronize()
+    one = max(c0.elapsed_time(c1), 1e-3)
+    n = int(min(max_reps, max(min_reps, math.ceil(min_seconds * 1e3 / one))))
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
+    torch.cuda.synchronize()
+    t0 = time.time()
+    evs[0].record(stream)
+    for i in range(n):
+        enqueue()
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    return [evs[i].elapsed_time(evs[i + 1]) for i in range(n)], t0, t1
 
-    if rank == 0:
-        zbuild.build()
-    if world > 1:
-        dist.barrier()
+
+def rep_stats(ms, K, dev, world):
+    """Median and minimum of the per-region times (max over ranks), per step."""
+    med = max_over_ranks(float(np.median(ms)), dev, world)
+    mn = max_over_ranks(float(np.min(ms)), dev, world)
+    return med / K, mn / K, len(ms)
+
+
+# The configurations reported in `per_config`: (entry, workload, mask mode
+# override). long_ctx runs in both of its modes; tiny_fp32 (both modes in its
+# parity tests) is timed in slot-causal mode.
+PER_CONFIG = [("tiny_fp32", "tiny_fp32", 1), ("decode_small", "decode_small", None),
+              ("ragged_mid", "ragged_mid", None), ("long_ctx_bidir", "long_ctx", 0),
+              ("long_ctx_causal", "long_ctx", 1), ("serving_mix", "serving_mix", None)]
+
+
+def entry_workload(entry):
+    for e, name, mode in PER_CONFIG:
+        if e == entry:
+            return name, mode
+    raise KeyError(entry)
+
+
+def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_seconds,
+                     cpu_budget, full, sampler_windows):
+    """Measures one configuration: the slot-decode step (staged attention +
+    length commit) over K steps, the attention launches alone, and the step
+    end to end through the public API with host buffers; each as repeated
+    K-step regions (median and minimum). With `full`, also the step with the
+    copying commit. Returns a dict (see run_ours)."""
+    import torch
+
     from paper_2609_19868_gb300 import _binding as zb
     from paper_2609_19868_gb300 import session
     from paper_2609_19868_gb300 import workloads as wl
 
-    zb.load()
-    zb.check_device_error()
+    name, mode = entry_workload(entry)
     # weak scaling: every rank runs its own batch (distinct seed)
-    seed = wl.SPECS[args.workload]["seed"] + 1000 * rank
-    w = wl.make(args.workload, seed=seed)
-    if w.both_modes:
-        w = w.with_mode(1)
+    seed = wl.SPECS[name]["seed"] + 1000 * rank
+    w = wl.make(name, seed=seed)
+    if mode is not None:
+        w = w.with_mode(mode)
     counts = algorithmic_counts(w)
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     cache_bytes = (w.k_cache.numel() + w.v_cache.numel()) * w.k_cache.element_size()
     n_rot = max(2, math.ceil(3 * l2 / max(cache_bytes, 1)))
-    stream = torch.cuda.Stream(dev)
     rots = []
     with torch.cuda.stream(stream):
         base = session.upload(w, dev)
         rots.append(base)
         for _ in range(n_rot - 1):
             kc, vc = base.k_cache.clone(), base.v_cache.clone()
-            db = session.upload(w, dev, caches=(kc, vc))
-            rots.append(db)
+            rots.append(session.upload(w, dev, caches=(kc, vc)))
     # The commit writes the advanced lengths into a second array (the
     # ping-pong a decoding loop would use), so every step starts from the same
     # prefix lengths: a stationary workload with no copy between steps.
@@ -297,7 +429,14 @@ def run_ours(args):
         db.stage_and_attend(stream)
         db.commit_staged(stream, new_lens=lens_next[id(db)])
 
-    K, W = args.steps, args.warmup
+    def attend(db):
+        db.attend(stream)
+
+    def step_copy(db):
+        # the same step with the commit copying the accepted rows again
+        db.stage_and_attend(stream)
+        db.commit(stream, new_lens=lens_next[id(db)])
+
     with torch.cuda.stream(stream):
         for i in range(max(W, n_rot)):
             step(rots[i % n_rot])
@@ -307,9 +446,8 @@ def run_ours(args):
     # CUDA graphs hold n_rot consecutive steps, one per cache rotation (as a
     # serving loop captures a whole forward pass): the kernels of successive
     # steps chain through programmatic dependent launch instead of paying a
-    # graph launch each. A tail graph with the first K % n_rot steps makes the
-    # timed region exactly K steps. The attention launches alone are captured
-    # the same way for the per-launch kernel time.
+    # graph launch each. A tail graph with the first K % n_rot steps makes each
+    # timed region exactly K steps.
     def capture(fn, count):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
@@ -317,78 +455,45 @@ def run_ours(args):
                 fn(rots[r])
         return g
 
-    def attend(db):
-        db.attend(stream)
-
     def capture_fn(fn):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             fn()
         return g
 
-    def step_copy(db):
-        # the same step with the commit copying the accepted rows again
-        db.stage_and_attend(stream)
-        db.commit(stream, new_lens=lens_next[id(db)])
+    full_n, tail = divmod(K, n_rot)
 
-    full, tail = divmod(K, n_rot)
-    step_graph = capture(step, n_rot)
-    step_tail = capture(step, tail) if tail else None
-    attn_graph = capture(attend, n_rot)
-    attn_tail = capture(attend, tail) if tail else None
-    copy_graph = capture(step_copy, n_rot)
-    copy_tail = capture(step_copy, tail) if tail else None
+    def region(graph, tail_graph):
+        def enqueue():
+            for _ in range(full_n):
+                graph.replay()
+            if tail_graph is not None:
+                tail_graph.replay()
+        return enqueue
 
-    def run(graph, tail_graph):
-        for _ in range(full):
-            graph.replay()
-        if tail_graph is not None:
-            tail_graph.replay()
-
-    for _ in range(max(1, -(-W // n_rot))):
-        step_graph.replay()
+    graphs = {"step": (capture(step, n_rot), capture(step, tail) if tail else None),
+              "attn": (capture(attend, n_rot), capture(attend, tail) if tail else None)}
+    if full:
+        graphs["copy"] = (capture(step_copy, n_rot), capture(step_copy, tail) if tail else None)
+    with torch.cuda.stream(stream):
+        for g, gt in graphs.values():
+            for _ in range(max(1, -(-W // n_rot))):
+                g.replay()
     torch.cuda.synchronize()
     assert zb.check_device_error(stream) == 0
 
-    sampler = ClockSampler(local).start() if args.clocks else None
-    if sampler:
-        time.sleep(0.3)
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    t0 = time.time()
+    res = {}
     with torch.cuda.stream(stream):
-        start.record(stream)
-        run(step_graph, step_tail)
-        end.record(stream)
+        for key, (g, gt) in graphs.items():
+            if world > 1:
+                import torch.distributed as dist
+
+                dist.barrier()
+            ms, t0, t1 = timed_reps(region(g, gt), stream, min_reps, min_seconds)
+            res[key] = rep_stats(ms, K, dev, world)
+            sampler_windows.append((entry, key, t0, t1))
     torch.cuda.synchronize()
-    t1 = time.time()
-    if world > 1:
-        dist.barrier()
-    total_ms = start.elapsed_time(end)
-    # Per-launch attention time: the same K launches back to back over the
-    # rotating caches (every launch reads its KV from HBM), CUDA events on the
-    # launching stream around the loop.
-    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        a0.record(stream)
-        run(attn_graph, attn_tail)
-        a1.record(stream)
-    torch.cuda.synchronize()
-    clocks = sampler.stop(t0, time.time()) if sampler else None
     assert zb.check_device_error(stream) == 0
-    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        c0.record(stream)
-        run(copy_graph, copy_tail)
-        c1.record(stream)
-    torch.cuda.synchronize()
-    copy_ms = max_over_ranks(c0.elapsed_time(c1) / K, dev, world)
-    attn_ms = max_over_ranks(a0.elapsed_time(a1) / K, dev, world)
-    attn_method = (f"{K} attention launches back to back ({n_rot} per CUDA graph, one per cache "
-                   "rotation), CUDA events on the launching stream")
-    total_ms = max_over_ranks(total_ms, dev, world)
 
     # End to end through the public API, every step: the step's inputs (q,
     # k_new, v_new, accept_len, packed in one pinned host buffer) copied to the
@@ -399,8 +504,8 @@ def run_ours(args):
     # rotation's copy-in, step and copy-out), as a serving loop would overlap
     # transfers with compute; the n_rot steps of a rotation cycle, copies
     # included, are one CUDA graph. (Copy-engine memcpy nodes in the same
-    # graph cost 28.6 us per step instead of 22.9: each hand-over between a
-    # memcpy node and the kernels around it takes microseconds.)
+    # graph cost several microseconds per hand-over between a memcpy node and
+    # the kernels around it.)
     def align(x):
         return (x + 255) // 256 * 256
 
@@ -421,10 +526,9 @@ def run_ours(args):
     for db in rots:
         buf = torch.empty(total, dtype=torch.uint8, device=dev)
         dev_in.append(buf)
-        for (name, t), o in zip(parts, offs):
+        for (nm, t), o in zip(parts, offs):
             nbytes = t.numel() * t.element_size()
-            view = buf[o:o + nbytes].view(t.dtype).view(t.shape)
-            setattr(db, name, view)
+            setattr(db, nm, buf[o:o + nbytes].view(t.dtype).view(t.shape))
     s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     ev_in = [torch.cuda.Event() for _ in rots]
     ev_done = [torch.cuda.Event() for _ in rots]
@@ -453,25 +557,133 @@ def run_ours(args):
     torch.cuda.synchronize()
     e2e_graph = capture_fn(lambda: e2e_steps(n_rot))
     e2e_tail = capture_fn(lambda: e2e_steps(tail)) if tail else None
-    for _ in range(max(1, -(-W // n_rot))):
-        e2e_graph.replay()
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, -(-W // n_rot))):
+            e2e_graph.replay()
     torch.cuda.synchronize()
     if world > 1:
+        import torch.distributed as dist
+
         dist.barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
-        e0.record(stream)
-        run(e2e_graph, e2e_tail)
-        e1.record(stream)
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    e2e_ms = max_over_ranks(e2e_ms, dev, world)
+        ms, t0, t1 = timed_reps(region(e2e_graph, e2e_tail), stream, min_reps, min_seconds)
+    sampler_windows.append((entry, "e2e", t0, t1))
+    res["e2e"] = rep_stats(ms, K, dev, world)
     assert zb.check_device_error(stream) == 0
 
     hbm_peak, tf_peak, peak_src = read_peaks()
-    attn_gbs = counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9
-    attn_tflops = counts["flops"] / (attn_ms * 1e-3) / 1e12
-    value = replica_throughput(K, world, total_ms)
+    attn_ms = res["attn"][0]
+    step_ms = res["step"][0]
+    out = {
+        "workload": WORKLOAD_LABELS[entry],
+        "w": w,
+        "counts": counts,
+        "n_rot": n_rot,
+        "cache_bytes": cache_bytes,
+        "l2": l2,
+        "step_ms": res["step"],
+        "attn_ms": res["attn"],
+        "copy_ms": res.get("copy"),
+        "e2e_ms": res["e2e"],
+        "h2d": int(h2d),
+        "d2h": int(d2h),
+        "roofline": roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src,
+                                          recorded_traffic(entry)),
+        "hbm_gbs": counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9,
+        "tflops": counts["flops"] / (attn_ms * 1e-3) / 1e12,
+        "steps_per_s": replica_throughput(K, world, step_ms * K),
+    }
+    del rots, graphs, e2e_graph, e2e_tail, dev_in, base
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and cpu_budget > 0:
+        out["cpu_baseline"] = cpu_baseline(w, budget_s=cpu_budget)
+    return out
+
+
+def config_entry(m, K, world):
+    """The per_config record of one measured configuration."""
+    (s_med, s_min, s_n), (a_med, a_min, a_n) = m["step_ms"], m["attn_ms"]
+    e_med, e_min, e_n = m["e2e_ms"]
+    c = m["counts"]
+    rec = {
+        "workload": m["workload"],
+        "ms_per_step": round(s_med, 5),
+        "ms_per_step_min": round(s_min, 5),
+        "steps_per_s": round(replica_throughput(K, world, s_med * K), 2),
+        "attn_ms_per_launch": round(a_med, 5),
+        "attn_ms_per_launch_min": round(a_min, 5),
+        "hbm_gbs": round(m["hbm_gbs"], 1),
+        "tflops": round(m["tflops"], 2),
+        "algorithmic_bytes": c["attn_bytes"],
+        "algorithmic_flops": c["flops"],
+        "roofline": m["roofline"],
+        "e2e": {"value": round(replica_throughput(K, world, e_med * K), 2), "unit": "steps/s",
+                "h2d_bytes_per_step": m["h2d"], "d2h_bytes_per_step": m["d2h"]},
+        "timing": f"{s_n} regions of {K} steps (median; min also given)",
+    }
+    if "cpu_baseline" in m:
+        rec["cpu_baseline"] = m["cpu_baseline"]
+    return rec
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    if rank == 0:
+        zbuild.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2609_19868_gb300 import _binding as zb
+
+    zb.load()
+    zb.check_device_error()
+    K, W = args.steps, args.warmup
+    stream = torch.cuda.Stream(dev)
+    sampler = ClockSampler(local).start() if args.clocks else None
+    if sampler:
+        time.sleep(0.3)
+    windows = []
+    head = measure_workload(args.workload, args, dev, stream, world, rank, K, W, args.reps,
+                            args.min_seconds, 0.0 if args.no_cpu_baseline else args.cpu_budget,
+                            True, windows)
+    per_config = {}
+    if args.per_config:
+        for entry, _, _ in PER_CONFIG:
+            if entry == args.workload:
+                m = head
+            else:
+                m = measure_workload(entry, args, dev, stream, world, rank, K, W,
+                                     args.reps, args.config_seconds,
+                                     0.0 if args.no_cpu_baseline else args.cpu_budget / 4,
+                                     False, windows)
+            per_config[entry] = config_entry(m, K, world)
+            if m is not head:
+                del m
+    clocks_all = None
+    if sampler:
+        step_win = [(t0, t1) for e, key, t0, t1 in windows if e == args.workload and key == "step"]
+        clocks = sampler.stop(*step_win[0], keep=True)
+        for entry in per_config:
+            wins = [(t0, t1) for e, key, t0, t1 in windows if e == entry]
+            per_config[entry]["clocks"] = sampler.window(wins[0][0], wins[-1][1])
+        clocks_all = sampler.window(windows[0][2], windows[-1][3])
+    else:
+        clocks = None
+
+    w = head["w"]
+    (s_med, s_min, s_n), (a_med, a_min, a_n) = head["step_ms"], head["attn_ms"]
+    e_med = head["e2e_ms"][0]
+    c_med = head["copy_ms"][0]
+    value = replica_throughput(K, world, s_med * K)
     line = {
         "metric": "slot-decode steps/s (one layer: stage + slot attention + commit)",
         "value": round(value, 2),
@@ -479,47 +691,54 @@ def run_ours(args):
         "n_gpus": world,
         "steps": K,
         "warmup": W,
-        "ms_per_step": round(total_ms / K, 5),
+        "ms_per_step": round(s_med, 5),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
+        "dtype": "bf16" if w.dtype == "bf16" else "f32",
         "data": "synthetic (seeded N(0,1), random-init; no weights or datasets)",
         "config": {
-            "workload": WORKLOAD_LABELS.get(args.workload, args.workload),
+            "workload": head["workload"],
             "global_batch": w.B * world,
-            "block_rows_per_seq": int(w.max_rows),
-            "kv_len": int((w.cache_lens + w.R).max()),
-            "l2": f"{n_rot} rotating KV caches of {cache_bytes / 1e6:.1f} MB "
-                  f"(> L2 {l2 / 1e6:.0f} MB between reuses)",
+            "block_rows_per_seq_max": int(w.max_rows),
+            "kv_len_max": int((w.cache_lens + w.R).max()),
+            "l2": f"{head['n_rot']} rotating KV caches of {head['cache_bytes'] / 1e6:.1f} MB "
+                  f"(> L2 {head['l2'] / 1e6:.0f} MB between reuses)",
             "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-            "launch": f"CUDA graphs of {n_rot} steps (programmatic dependent launch between kernels)",
+            "launch": f"CUDA graphs of {head['n_rot']} steps (programmatic dependent launch "
+                      "between kernels)",
         },
+        "timing": {"regions": s_n, "steps_per_region": K, "statistic": "median region",
+                   "ms_per_step_min": round(s_min, 5),
+                   "method": "CUDA events between back-to-back K-step regions on the "
+                             "launching stream; max over ranks"},
         "attn": {
-            "ms_per_launch": round(attn_ms, 5),
-            "timing": attn_method,
-            "hbm_gbs": round(attn_gbs, 1),
-            "tflops": round(attn_tflops, 2),
-            "algorithmic_bytes": counts["attn_bytes"],
-            "algorithmic_flops": counts["flops"],
+            "ms_per_launch": round(a_med, 5),
+            "ms_per_launch_min": round(a_min, 5),
+            "timing": f"{a_n} regions of {K} attention launches back to back ({head['n_rot']} per "
+                      "CUDA graph, one per cache rotation), CUDA events on the launching stream; "
+                      "median region",
+            "hbm_gbs": round(head["hbm_gbs"], 1),
+            "tflops": round(head["tflops"], 2),
+            "algorithmic_bytes": head["counts"]["attn_bytes"],
+            "algorithmic_flops": head["counts"]["flops"],
         },
-        "roofline": roofline_entry(counts, attn_gbs, attn_tflops, hbm_peak, tf_peak, peak_src,
-                                   recorded_traffic(args.workload)),
+        "roofline": head["roofline"],
         "e2e": {
-            "value": round(replica_throughput(K, world, e2e_ms), 2),
+            "value": round(replica_throughput(K, world, e_med * K), 2),
             "unit": "steps/s",
-            "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h),
+            "h2d_bytes_per_step": head["h2d"],
+            "d2h_bytes_per_step": head["d2h"],
             "transfers": "zarya_copy kernels through the pinned buffers' device mapping, "
                          "on side streams pipelined with the steps (one CUDA graph per "
                          "rotation cycle)",
         },
         "step_forms": {
-            "commit_staged": {"ms_per_step": round(total_ms / K, 5),
+            "commit_staged": {"ms_per_step": round(s_med, 5),
                               "note": "zarya_slot_attn_staged + zarya_kv_commit_staged (the "
                                       "accepted rows are already in place: lengths advance)"},
-            "commit_copy": {"ms_per_step": round(copy_ms, 5),
-                            "steps_per_s": round(replica_throughput(K, world, copy_ms * K), 2),
+            "commit_copy": {"ms_per_step": round(c_med, 5),
+                            "steps_per_s": round(replica_throughput(K, world, c_med * K), 2),
                             "note": "zarya_slot_attn_staged + zarya_kv_append_commit_to (the "
                                     "accepted rows copied again)"},
         },
@@ -528,11 +747,17 @@ def run_ours(args):
             "layers_28_steps_per_s": round(value / 28, 2),
             "layers_36_steps_per_s": round(value / 36, 2),
         },
-        "gpu_launches": 2 * K,   # staged attention, commit (length advance)
+        # staged attention + length commit per step, in every timed region
+        "gpu_launches": 2 * K * s_n,
+        "gpu_launches_note": f"2 kernels per step x {K} steps x {s_n} timed regions",
         "clocks": clocks,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    if per_config:
+        line["per_config"] = per_config
+        if clocks_all is not None:
+            line["clocks_whole_run"] = clocks_all
+    if "cpu_baseline" in head:
+        line["cpu_baseline"] = head["cpu_baseline"]
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -1038,8 +1263,9 @@ def select_cpu_baseline(w, T, sb, budget_s=20.0):
                       f"(numpy fp64 oracle), scaled to the whole step by rows"}
 
 
-def _oracle_step(oracle, w, seqs, threads=0):
-    """The oracle's version of one step restricted to sequences ``seqs``."""
+def workload_subset(w, seqs):
+    """The workload restricted to sequences ``seqs`` (their rows, lengths and
+    caches; a paged cache keeps only their pages, renumbered)."""
     from dataclasses import replace
 
     sub = w
@@ -1052,13 +1278,28 @@ def _oracle_step(oracle, w, seqs, threads=0):
 
         ridx = torch.as_tensor(rows)
         if w.page_size:
-            raise ValueError("subsets of paged workloads are not used")
+            # the subset's own pages, renumbered into a compact pool
+            table = w.page_table[idx]
+            used = np.unique(table[table >= 0])
+            remap = np.full(w.n_pages, -1, dtype=np.int64)
+            remap[used] = np.arange(len(used))
+            new_table = np.where(table >= 0, remap[np.maximum(table, 0)], -1).astype(np.int32)
+            pidx = torch.as_tensor(used)
+            caches = dict(k_cache=w.k_cache[pidx], v_cache=w.v_cache[pidx],
+                          page_table=new_table, n_pages=len(used))
+        else:
+            caches = dict(k_cache=w.k_cache[torch.as_tensor(idx)],
+                          v_cache=w.v_cache[torch.as_tensor(idx)])
         sub = replace(w, B=len(idx), cache_lens=w.cache_lens[idx], n_slots=w.n_slots[idx],
                       slot_len=w.slot_len[idx], mask_mode=w.mask_mode[idx],
                       accept_len=w.accept_len[idx], q_row_offsets=new_offs,
-                      q=w.q[ridx], k_new=w.k_new[ridx], v_new=w.v_new[ridx],
-                      k_cache=w.k_cache[torch.as_tensor(idx)],
-                      v_cache=w.v_cache[torch.as_tensor(idx)])
+                      q=w.q[ridx], k_new=w.k_new[ridx], v_new=w.v_new[ridx], **caches)
+    return sub
+
+
+def _oracle_step(oracle, w, seqs, threads=0):
+    """The oracle's version of one step restricted to sequences ``seqs``."""
+    sub = workload_subset(w, seqs)
     t0 = time.perf_counter()
     kc, vc, lens = oracle.kv_append(sub.k_new, sub.v_new, sub.R, sub.k_cache, sub.v_cache,
                                     sub.cache_lens, sub.page_table, sub.q_row_offsets,
@@ -1072,22 +1313,33 @@ def _oracle_step(oracle, w, seqs, threads=0):
     return time.perf_counter() - t0
 
 
+def _visible_pairs(w):
+    """Visible (row, head, key) pairs of every sequence: the oracle's work."""
+    P = w.cache_lens.astype(np.int64)
+    R = w.R
+    return np.where(w.mask_mode == 0, w.Hq * R * (P + R), w.Hq * (R * P + R * (R + 1) // 2))
+
+
 def cpu_baseline(w, budget_s=20.0):
-    """The oracle, as it stands, on the host cores: whole steps over a subset
-    of the batch's sequences, scaled to the full batch."""
+    """The oracle, as it stands, on the host cores: whole steps over the
+    first sequences of the batch, scaled to the full batch by the visible
+    (row, head, key) pairs (the oracle's work is proportional to them)."""
     import oracle
 
     oracle.build()
     cores = oracle.max_threads()
+    pairs = _visible_pairs(w)
     t1 = _oracle_step(oracle, w, [0])
-    per_seq = t1
-    n_seq = int(max(1, min(w.B, budget_s / max(per_seq, 1e-6))))
+    per_pair = t1 / max(int(pairs[0]), 1)
+    n_seq = int(np.searchsorted(np.cumsum(pairs), budget_s / max(per_pair, 1e-15), side="right"))
+    n_seq = max(1, min(w.B, n_seq))
     t = _oracle_step(oracle, w, list(range(n_seq)))
-    step_s = t * w.B / n_seq
+    step_s = t * float(pairs.sum()) / float(pairs[:n_seq].sum())
     return {"value": round(1.0 / step_s, 4), "unit": "steps/s", "cores": cores,
             "kind": "oracle",
             "sample": f"{n_seq} of {w.B} sequences of one step (stage + attention + commit, "
-                      f"fp64 C oracle with OpenMP), scaled to the full batch"}
+                      f"fp64 C oracle with OpenMP, {t:.1f} s), scaled to the full batch by "
+                      f"visible (row, head, key) pairs"}
 
 
 def run_reference(args):
@@ -1099,23 +1351,26 @@ def run_reference(args):
     from paper_2609_19868_gb300 import workloads as wl
 
     oracle.build()
-    w = wl.make(args.workload)
-    if w.both_modes:
-        w = w.with_mode(1)
+    name, mode = entry_workload(args.workload)
+    w = wl.make(name)
+    if mode is not None:
+        w = w.with_mode(mode)
     cores = oracle.max_threads()
     # size each step's sample so the whole run stays within ~2 minutes
-    per_seq = _oracle_step(oracle, w, [0])
+    pairs = _visible_pairs(w)
+    per_pair = _oracle_step(oracle, w, [0]) / max(int(pairs[0]), 1)
     budget = 120.0 / max(1, args.steps + args.warmup)
-    n_seq = int(max(1, min(w.B, budget / max(per_seq, 1e-6))))
+    n_seq = int(np.searchsorted(np.cumsum(pairs), budget / max(per_pair, 1e-15), side="right"))
+    n_seq = max(1, min(w.B, n_seq))
     for _ in range(args.warmup):
         _oracle_step(oracle, w, list(range(n_seq)))
     total = 0.0
     for _ in range(args.steps):
         total += _oracle_step(oracle, w, list(range(n_seq)))
-    step_s = total / args.steps * w.B / n_seq
+    step_s = total / args.steps * float(pairs.sum()) / float(pairs[:n_seq].sum())
     value = 1.0 / step_s
     sample = (f"{n_seq} of {w.B} sequences per step (stage + attention + commit), "
-              f"scaled to the full batch")
+              f"scaled to the full batch by visible (row, head, key) pairs")
     line = {
         "impl": "reference",
         "metric": "slot-decode steps/s (one layer: stage + slot attention + commit)",
@@ -1195,11 +1450,19 @@ def run_select_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=None,
-                    choices=list(WORKLOAD_LABELS) + list(SELECT_LABELS))
+                    choices=list(WORKLOAD_LABELS) + list(WORKLOAD_ALIASES) + list(SELECT_LABELS))
+    ap.add_argument("--reps", type=int, default=30,
+                    help="at least this many timed K-step regions (median and min reported)")
+    ap.add_argument("--min-seconds", type=float, default=1.0,
+                    help="the headline's repeated regions last at least this long")
+    ap.add_argument("--config-seconds", type=float, default=0.3,
+                    help="each per_config entry's repeated regions last at least this long")
+    ap.add_argument("--no-per-config", dest="per_config", action="store_false",
+                    help="measure the chosen workload only")
     ap.add_argument("--path", choices=["attention", "select", "reorder", "mode_a"],
                     default="attention",
                     help="attention: the slot-decode layer step (stage + attention + commit); "
@@ -1212,7 +1475,10 @@ def main():
     if args.warmup < 3:
         args.warmup = 3
     if args.workload is None:
-        args.workload = "select_decode_small" if args.path == "select" else "decode_small"
+        args.workload = "select_decode_small" if args.path == "select" else "serving_mix"
+    args.workload = WORKLOAD_ALIASES.get(args.workload, args.workload)
+    if args.path == "attention" and args.workload not in WORKLOAD_LABELS:
+        ap.error(f"--workload {args.workload} is not an attention workload")
     if args.path == "mode_a":
         if args.impl == "reference":
             print(json.dumps({"impl": "reference", "unavailable":

@@ -34,6 +34,11 @@
  *    out) set a per-device error word; the affected work is skipped, never
  *    trapped. Read (and clear) it with zarya_check_device_error.
  *  - bf16 tensors use round-to-nearest-even on output; fp32 accumulation.
+ *  - The library keeps per-device set-up for the life of the process: the
+ *    device addresses of its error word and of the zarya_slot_attn_noalloc
+ *    scratch, and kernel attributes. Do not call it on a device after
+ *    cudaDeviceReset there: the cached addresses would point into the
+ *    destroyed context.
  */
 #ifndef ZARYA_H_
 #define ZARYA_H_

@@ -54,13 +54,22 @@ _F64, _F32, _BF16 = 0, 1, 2
 
 def build(force: bool = False) -> str:
     """Compile the C oracle with gcc + OpenMP into ``oracle/liboracle.so``."""
-    if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
-        return _LIB_PATH
+    import hashlib
+
+    cmd_flags = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp"]
+    with open(_SRC, "rb") as f:
+        digest = hashlib.sha256(" ".join(cmd_flags).encode() + b"\0" + f.read()).hexdigest()
+    stamp = _LIB_PATH + ".sha256"
+    if not force and os.path.exists(_LIB_PATH) and os.path.exists(stamp):
+        with open(stamp) as f:
+            if f.read().strip() == digest:
+                return _LIB_PATH
     tmp = _LIB_PATH + ".tmp%d" % os.getpid()
-    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-o", tmp, _SRC, "-lm"]
-    subprocess.run(cmd, check=True)
+    subprocess.run(cmd_flags + ["-o", tmp, _SRC, "-lm"], check=True)
     os.replace(tmp, _LIB_PATH)
+    with open(stamp + ".tmp", "w") as f:
+        f.write(digest + "\n")
+    os.replace(stamp + ".tmp", stamp)
     return _LIB_PATH
 
 

@@ -41,16 +41,37 @@ def _inputs():
     return files
 
 
+STAMP = LIB + ".sha256"
+
+
+def source_digest() -> str:
+    """SHA-256 over the build's inputs (sources, headers, nvcc flags), in a
+    fixed order: the library is rebuilt whenever any of them changes,
+    whatever the files' modification times say."""
+    import hashlib
+
+    h = hashlib.sha256()
+    h.update(" ".join(ARCH + FLAGS[:-4]).encode())
+    for f in sorted(_inputs()):
+        h.update(os.path.basename(f).encode() + b"\0")
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+    """True when libzarya.so exists and was linked from the current sources
+    (the digest recorded beside it at link time matches)."""
+    if not os.path.exists(LIB) or not os.path.exists(STAMP):
         return False
-    t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(f) <= t for f in _inputs())
+    with open(STAMP) as f:
+        return f.read().strip() == source_digest()
 
 
 def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
     if not force and up_to_date():
         return LIB
+    digest = source_digest()
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
     extra = ["-Xptxas", "-v"] if ptxas_info else []
@@ -76,6 +97,9 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
     os.replace(tmp, LIB)
+    with open(STAMP + ".tmp", "w") as f:
+        f.write(digest + "\n")
+    os.replace(STAMP + ".tmp", STAMP)
     return LIB
 
 

@@ -73,7 +73,9 @@ zarya_status zarya_slot_attn_noalloc(const void* q, const void* k_cache, const v
     // The split counters sit at the end of the workspace layout and must
     // start at zero; the array keeps whatever the last call left.
     const size_t cnt_bytes = zarya::workspace_counter_bytes(desc);
-    if (cnt_bytes == 0 || cnt_bytes > need) return ZARYA_ERR_CUDA;
+    if (cnt_bytes == 0 || cnt_bytes > need)
+      return zarya::cuda_fail("split counter layout does not fit the scratch plan",
+                              cudaErrorInvalidValue);
     ce = cudaMemsetAsync(static_cast<unsigned char*>(scratch) + (need - cnt_bytes), 0, cnt_bytes,
                          stream);
     if (ce != cudaSuccess) return zarya::cuda_fail("clearing the split counters", ce);

@@ -310,6 +310,8 @@ def test_repetition_penalty_rejects_invalid_calls(lib):
     assert call(d=None) == 1
     assert call(d=_sdesc(vocab=0)) == 1
     assert call(d=_sdesc(vocab=2_000_000, row_stride=2_000_000)) == 2   # bitmap too large
+    # rows closer together than the vocabulary would overlap (and be penalised twice)
+    assert call(d=_sdesc(vocab=1000, row_stride=992)) == 1
 
 
 def test_top_p_rejects_invalid_calls(lib):
@@ -321,3 +323,6 @@ def test_top_p_rejects_invalid_calls(lib):
         assert lib.zarya_top_p(vp(FAKE), p, ctypes.byref(d), None) == 1
     assert lib.zarya_top_p(vp(FAKE), 0.9, None, None) == 1
     assert lib.zarya_top_p(vp(FAKE), 1.0, ctypes.byref(d), None) == 0   # nothing to cut
+    # overlapping rows (stride below the vocabulary) are refused before anything runs
+    short = _sdesc(vocab=1000, row_stride=992)
+    assert lib.zarya_top_p(vp(FAKE), 0.9, ctypes.byref(short), None) == 1

@@ -39,3 +39,77 @@ def test_alu_roofline_counts_philox_multiplies():
     assert e["achieved"] == pytest.approx(achieved, abs=0.1)
     assert e["frac"] == pytest.approx(achieved / e["peak"], abs=1e-4)
     assert e["algorithmic_muls"] == 10 * n_logits
+
+
+def _uniform_workload(mode):
+    from paper_2609_19868_gb300 import workloads as wl
+
+    return wl.make("decode_small", small=True).with_mode(mode)
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+def test_per_sequence_roofline_of_a_uniform_batch_is_the_single_intensity_one(mode):
+    """Every sequence of decode_small has the same shape, so the per-sequence
+    ideal time is the batch's bytes / HBM (or flops / bf16), whichever is
+    larger, and the entry's peak is the measured one."""
+    w = _uniform_workload(mode)
+    c = bench.algorithmic_counts(w)
+    ideal, hbm, tc, wide = bench.per_sequence_roofline(w, 6691.1, 1926.3)
+    assert ideal == pytest.approx(max(c["attn_bytes"] / 6691.1e9, c["flops"] / 1926.3e12))
+    assert ideal == pytest.approx(wide)
+    e = bench.roofline_per_sequence(w, c, attn_ms=ideal * 1e3 * 2, hbm_peak=6691.1,
+                                    tf_peak=1926.3, peak_src="measured", traffic=None)
+    assert e["peak"] in (6691.1, 1926.3)
+    assert e["frac"] == pytest.approx(0.5, abs=1e-4)
+
+
+def test_per_sequence_roofline_of_a_mixed_batch():
+    """Hand-built two-sequence batch: one sequence is HBM-bound (a long prefix
+    read by 4 rows), the other tensor-bound (a short prefix read by 512 rows).
+    The ideal time is the sum of their own bounds, which is at least the
+    batch-wide max(bytes / HBM, flops / bf16), and frac = ideal / measured."""
+    from dataclasses import replace
+
+    import numpy as np
+
+    w = _uniform_workload(1)
+    w = replace(w, B=2, cache_lens=np.array([16384, 1024], np.int32),
+                n_slots=np.array([1, 16], np.int32), slot_len=np.array([4, 32], np.int32),
+                mask_mode=np.array([1, 0], np.int32), Hq=32, Hkv=8, D=128,
+                q_row_offsets=np.array([0, 4, 516], np.int32))
+    hbm_gbs, tf = 6691.1, 1926.3
+    P = np.array([16384, 1024]); R = np.array([4, 512])
+    byts = 8 * (P + R) * 128 * 2 * 2 + 2 * R * 32 * 128 * 2
+    pairs = np.array([32 * (4 * 16384 + 4 * 5 // 2), 32 * 512 * (1024 + 512)])
+    flops = 4 * 128 * pairs
+    t_h, t_t = byts / (hbm_gbs * 1e9), flops / (tf * 1e12)
+    assert t_h[0] > t_t[0] and t_t[1] > t_h[1]
+    ideal, hbm, tc, wide = bench.per_sequence_roofline(w, hbm_gbs, tf)
+    assert ideal == pytest.approx(t_h[0] + t_t[1])
+    assert hbm == pytest.approx(t_h[0]) and tc == pytest.approx(t_t[1])
+    assert wide == pytest.approx(max(byts.sum() / (hbm_gbs * 1e9), flops.sum() / (tf * 1e12)))
+    assert wide <= ideal
+    c = {"attn_bytes": int(byts.sum()), "flops": int(flops.sum())}
+    e = bench.roofline_per_sequence(w, c, attn_ms=ideal * 1e3 / 0.8, hbm_peak=hbm_gbs,
+                                    tf_peak=tf, peak_src="measured", traffic=None)
+    assert e["frac"] == pytest.approx(0.8, abs=1e-4)
+    assert e["achieved"] / e["peak"] == pytest.approx(e["frac"], abs=1e-3)
+    assert e["peak_measured"] == (tf if e["bound"] == "tensor" else hbm_gbs)
+
+
+def test_paged_subset_keeps_each_sequences_attention(oracle_mod):
+    """bench's oracle samples of a paged batch keep only the sampled
+    sequences' pages, renumbered: their attention must be unchanged."""
+    import numpy as np
+
+    from _helpers import oracle_full, oracle_staged
+    from paper_2609_19868_gb300 import workloads as wl
+
+    w = wl.make("serving_mix", small=True, B=4)
+    full = oracle_full(oracle_mod, w, *oracle_staged(oracle_mod, w))
+    sub = bench.workload_subset(w, [0, 2])
+    assert sub.n_pages < w.n_pages
+    got = oracle_full(oracle_mod, sub, *oracle_staged(oracle_mod, sub))
+    offs = w.q_row_offsets
+    want = np.concatenate([full[offs[0]:offs[1]], full[offs[2]:offs[3]]])
+    assert np.array_equal(got, want)
