@@ -88,7 +88,8 @@ typedef enum { ZARYA_BF16 = 0, ZARYA_FP32 = 1 } zarya_dtype;
 #define ZARYA_DEVERR_ROWS 2           /* R_b > max_rows, or q_row_offsets inconsistent with R_b */
 #define ZARYA_DEVERR_CAPACITY 3       /* P_b + rows would pass cache_capacity */
 #define ZARYA_DEVERR_ACCEPT 4         /* accept_len[b] outside [0, R_b] */
-#define ZARYA_DEVERR_TIMEOUT 5        /* a pipeline wait gave up (no progress for ~2 s) */
+#define ZARYA_DEVERR_TIMEOUT 5        /* a pipeline wait gave up (no progress for
+                                         desc->wait_limit_us, 2 s by default) */
 #define ZARYA_DEVERR_MASK_MODE 6      /* mask_mode[b] not a zarya_mask_mode */
 #define ZARYA_DEVERR_TOKEN 7          /* a verification token outside [0, vocab) */
 #define ZARYA_DEVERR_PERM 8           /* a permutation entry outside [0, lens[b]) */
@@ -112,7 +113,20 @@ typedef struct {
   float scale;             /* softmax scale; 0 means 1 / sqrt(D) */
   const int32_t* q_row_offsets; /* device [B + 1]: first row of sequence b in q / out /
                                    k_new; q_row_offsets[b+1] - q_row_offsets[b] == R_b */
+  int32_t wait_limit_us;   /* bound on every pipeline wait of the tensor-core attention kernel,
+                              in microseconds of global time; 0 = 2,000,000 (2 s). A wait that
+                              runs out sets ZARYA_DEVERR_TIMEOUT and its CTA unwinds (lets its
+                              own copies and MMAs finish, frees its tensor memory, writes no
+                              output). A failure-detection knob: normal waits last microseconds. */
+  int32_t debug_flags;     /* 0 in normal use; ZARYA_DEBUG_STALL tests the timeout path */
 } zarya_attn_desc;
+
+/* zarya_attn_desc.debug_flags: the tensor-core attention kernel's MMA warp
+ * first waits on a barrier that nothing completes, so that wait runs out after
+ * wait_limit_us and the launch unwinds with ZARYA_DEVERR_TIMEOUT, leaving the
+ * device usable (used by tests of the failure path; with kv_splits = 1 or
+ * more than 3, i.e. no thread-block cluster merge). */
+#define ZARYA_DEBUG_STALL 1
 
 /*
  * Bytes of scratch memory zarya_slot_attn needs for `desc` (0 if it needs

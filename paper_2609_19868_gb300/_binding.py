@@ -23,6 +23,8 @@ BF16, FP32 = 0, 1
 APPEND_STAGE, APPEND_COMMIT = 0, 1
 DEVERR_NAMES = {0: "none", 1: "page id", 2: "rows", 3: "capacity", 4: "accept length",
                 5: "timeout", 6: "mask mode"}
+DEVERR_TIMEOUT = 5
+DEBUG_STALL = 1
 
 
 class ZaryaError(RuntimeError):
@@ -51,6 +53,8 @@ class AttnDesc(ctypes.Structure):
         ("kv_splits", ctypes.c_int32),
         ("scale", ctypes.c_float),
         ("q_row_offsets", ctypes.c_void_p),
+        ("wait_limit_us", ctypes.c_int32),
+        ("debug_flags", ctypes.c_int32),
     ]
 
 
@@ -176,13 +180,15 @@ def _check_cuda(name: str, t: torch.Tensor, dtype=None):
 def make_desc(*, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int, dtype: int,
               page_size: int, cache_capacity: int, n_pages: int, max_rows: int,
               total_rows: int, q_row_offsets: torch.Tensor, max_kv_len: int = 0,
-              kv_splits: int = 0, scale: float = 0.0) -> AttnDesc:
+              kv_splits: int = 0, scale: float = 0.0, wait_limit_us: int = 0,
+              debug_flags: int = 0) -> AttnDesc:
     _check_cuda("q_row_offsets", q_row_offsets, torch.int32)
     d = AttnDesc()
     d.batch, d.n_q_heads, d.n_kv_heads, d.head_dim = batch, n_q_heads, n_kv_heads, head_dim
     d.dtype, d.page_size, d.cache_capacity, d.n_pages = dtype, page_size, cache_capacity, n_pages
     d.max_rows, d.total_rows, d.max_kv_len, d.kv_splits = max_rows, total_rows, max_kv_len, kv_splits
     d.scale = scale
+    d.wait_limit_us, d.debug_flags = wait_limit_us, debug_flags
     d.q_row_offsets = q_row_offsets.data_ptr()
     d._keep = q_row_offsets  # keep the offsets alive as long as the descriptor
     return d

@@ -57,6 +57,8 @@ zarya_status check_desc(const zarya_attn_desc* d) {
     return ZARYA_ERR_INVALID_ARG;
   if (!(d->scale >= 0.f) || std::isinf(d->scale)) return ZARYA_ERR_INVALID_ARG;
   if (d->q_row_offsets == nullptr) return ZARYA_ERR_INVALID_ARG;
+  if (d->wait_limit_us < 0 || (d->debug_flags & ~ZARYA_DEBUG_STALL) != 0)
+    return ZARYA_ERR_INVALID_ARG;
   if (d->page_size > 0) {
     if (d->cache_capacity % d->page_size != 0 || d->n_pages < 1) return ZARYA_ERR_INVALID_ARG;
   }
@@ -349,6 +351,9 @@ zarya_status slot_attn_impl(const void* q, const void* k_new, const void* v_new,
   p.splits = plan.splits;
   p.cluster = (plan.splits > 1 && plan.splits <= kMaxClusterSplits) ? 1 : 0;
   p.scale_log2 = scale * 1.4426950408889634f;
+  p.wait_ns = desc->wait_limit_us > 0 ? static_cast<uint64_t>(desc->wait_limit_us) * 1000ull
+                                       : 2000000000ull;
+  p.debug_stall = (desc->debug_flags & ZARYA_DEBUG_STALL) ? 1 : 0;
   p.k_new = k_new;
   p.v_new = v_new;
   p.k_cache = const_cast<void*>(k_cache);

@@ -38,6 +38,8 @@ struct TcParams {
   int m_tiles, splits;
   int cluster;        // 1: the splits of a tile form a cluster and merge through DSMEM
   float scale_log2;   // softmax scale * log2(e)
+  uint64_t wait_ns;   // bound on every pipeline wait (global-timer nanoseconds)
+  int debug_stall;    // 1: the MMA warp first waits on a barrier nothing completes
   // Staged attention: when k_new != nullptr, block row i of sequence b
   // (k_new / v_new row q_row_offsets[b] + i) is first written to cache
   // position P_b + i by the CTAs that read it.

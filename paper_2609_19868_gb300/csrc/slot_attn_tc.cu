@@ -38,9 +38,10 @@
 // tiles), warps 8-11 softmax group 1 (odd tiles). Warp w reads TMEM lanes
 // 32*(w%4) .. +31, i.e. the packed rows of that range.
 //
-// Every mbarrier wait is bounded (about 2 s of global time); a wait that
-// gives up records ZARYA_DEVERR_TIMEOUT, raises a CTA-wide abort flag and the
-// CTA unwinds (draining its own copies and MMAs, freeing TMEM).
+// Every mbarrier wait is bounded (p.wait_ns of global time, 2 s unless the
+// caller sets another limit); a wait that gives up records
+// ZARYA_DEVERR_TIMEOUT, raises a CTA-wide abort flag and the CTA unwinds
+// (draining its own copies and MMAs, freeing TMEM).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -65,7 +66,6 @@ constexpr uint32_t kOffV = kOffK + kStagesK * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kStagesV * kTileBytes;
 constexpr uint32_t kTmemCols = 512;  // S0/P0 [0,128) S1/P1 [128,256) O0 [256,384) O1 [384,512)
 constexpr uint32_t kTmemO = 256;
-constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
 constexpr uint64_t kDrainNs = 100000000ull;  // 100 ms
 
 struct Bars {
@@ -83,6 +83,7 @@ struct Bars {
   uint64_t stage_issued;  // staged attention: the first round of staging loads is issued
   uint64_t ready;   // cluster merge: every partial row this CTA owns has landed
   uint64_t go;      // cluster merge: every other split's K ring is free to receive
+  uint64_t stall;   // never completed: the debug stall waits on it until its limit
   uint32_t tmem_base;
   int abort;
   int last;
@@ -114,10 +115,9 @@ __device__ __forceinline__ void named_bar_arrive(int id, int n) {
 }
 
 // Named barriers (barrier 0 is __syncthreads): 1 joins the 256 softmax
-// threads, 2-5 one quadrant's warp of each softmax group, 6 the two producer
-// warps at entry, 7 publishes the entry set-up to the other ten warps.
+// threads, 2-5 one quadrant's warp of each softmax group, 7 publishes the
+// entry set-up to the other ten warps.
 constexpr int kBarSoftmax = 1;
-constexpr int kBarProducers = 6;
 constexpr int kBarSetup = 7;
 
 __device__ __forceinline__ void set_abort(Bars* bars, int* err, int code) {
@@ -125,9 +125,11 @@ __device__ __forceinline__ void set_abort(Bars* bars, int* err, int code) {
   *reinterpret_cast<volatile int*>(&bars->abort) = 1;
 }
 
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Bars* bars, int* err) {
-  if (mbar_wait(bar, parity, kWaitNs, &bars->abort)) return true;
-  set_abort(bars, err, ZARYA_DEVERR_TIMEOUT);
+// Bounded wait (p.wait_ns of global time) for a phase of a barrier of this CTA.
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Bars* bars,
+                                         const TcParams& p) {
+  if (mbar_wait(bar, parity, p.wait_ns, &bars->abort)) return true;
+  set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
   return false;
 }
 
@@ -232,9 +234,9 @@ __device__ __forceinline__ void cluster_merge_store(const float (&o)[64], float 
 // Bounded wait (acquire at cluster scope) for a phase completed by other CTAs
 // of the cluster.
 __device__ __forceinline__ bool wait_bar_cluster(uint64_t* bar, uint32_t parity, Bars* bars,
-                                                 int* err) {
-  if (mbar_wait_cluster(bar, parity, kWaitNs, &bars->abort)) return true;
-  set_abort(bars, err, ZARYA_DEVERR_TIMEOUT);
+                                                 const TcParams& p) {
+  if (mbar_wait_cluster(bar, parity, p.wait_ns, &bars->abort)) return true;
+  set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
   return false;
 }
 
@@ -330,7 +332,7 @@ __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* 
   const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
   for (int i = i_begin; i < i_end; ++i) {
     const int t = t_begin + i;
-    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p.err)) return false;
+    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p)) return false;
     int page = -1;
     uint32_t bytes = kTileBytes;
     if (paged) {
@@ -350,7 +352,7 @@ __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* 
     const int s = i % stages;
     bool w = true;
     if (lane == 0) {
-      w = wait_bar(&empty[s], ((i / stages) & 1) ^ 1, bars, p.err);
+      w = wait_bar(&empty[s], ((i / stages) & 1) ^ 1, bars, p);
       if (w) mbar_arrive_expect_tx(&full[s], bytes);
     }
     if (!__shfl_sync(0xffffffffu, w, 0)) return false;
@@ -457,18 +459,21 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     mbar_init(&bars->kfree, 1);
     mbar_init(&bars->staged, kSoftmaxWarps);
     mbar_init(&bars->stage_issued, kSoftmaxWarps);
+    mbar_init(&bars->stall, 1);
     bars->abort = 0;
     bars->last = 0;
     fence_mbar_init();
   }
+  // Every barrier is initialised before any thread touches one. The softmax
+  // warps signal stage_issued before the CTA-wide set-up barrier below, so
+  // without this barrier their arrive could land before thread 0's
+  // initialisation and be lost, and the producers' wait for it would run out.
+  // No copy is in flight yet, so nothing holds a thread here.
+  __syncthreads();
   // The producer warps load before the CTA-wide set-up barrier (a thread
-  // with tensor copies in flight waits for them at a barrier): they only sync
-  // with each other here and arrive, without waiting, on the set-up barrier
-  // the other ten warps wait on.
-  if (warp == 0 || warp == 2) {
-    named_bar_sync(kBarProducers, 64);
-    named_bar_arrive(kBarSetup, kThreads);
-  }
+  // with tensor copies in flight waits for them at a barrier): they arrive,
+  // without waiting, on the set-up barrier the other ten warps wait on.
+  if (warp == 0 || warp == 2) named_bar_arrive(kBarSetup, kThreads);
   // Before waiting for the kernel launched before this one, warm L2 with Q
   // and the first tiles of this split's K / V. L2 is the point of coherence,
   // so a prefetch cannot hand stale data to the loads made after the wait;
@@ -554,7 +559,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   if ((warp == 0 || warp == 2) && works) {
     if (stage_here) {
       // a timeout sets the abort flag; the ring loop below then returns early
-      if (lane == 0) wait_bar(&bars->stage_issued, 0, bars, p.err);
+      if (lane == 0) wait_bar(&bars->stage_issued, 0, bars, p);
       __syncwarp();
     }
     const bool is_k = warp == 0;
@@ -582,6 +587,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   // producer warps never use it.
   const uint32_t tmem = (warp != 0 && warp != 2) ? bars->tmem_base : 0u;
   bool cwaited = false;
+  bool mma_issued = false;   // the MMA warp issued at least one tcgen05.mma
   // Exits here are uniform over a cluster (its CTAs share the sequence and
   // M-tile and differ only in the split) or leave a split with no keys.
   if (!works) {
@@ -610,7 +616,11 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       // ======================= MMA issuer (one elected lane) =======================
       // The whole warp walks the issue loop (waits and descriptors are
       // warp-uniform); elect.sync picks the lane that issues MMAs and commits.
-      bool ok = wait_bar(&bars->q_full, 0, bars, p.err);
+      bool ok = true;
+      // Failure-path test: a wait that nothing completes runs out after
+      // p.wait_ns and the CTA unwinds like after any other timeout.
+      if (p.debug_stall) ok = wait_bar(&bars->stall, 0, bars, p);
+      if (ok) ok = wait_bar(&bars->q_full, 0, bars, p);
       bool any_mma = false;
       tc_fence_after();
       const uint64_t q_desc0 = sdesc_sw128(smem_u32(smem + kOffQ), 16, 1024);
@@ -622,7 +632,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       auto issue_qk = [&](int i) -> bool {
         const int s = i % kStagesK;
         const int sb = i & 1;
-        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p.err)) return false;
+        if (!wait_bar(&bars->k_full[s], (i / kStagesK) & 1, bars, p)) return false;
         tc_fence_after();
         const uint64_t kd = k_desc0 + s * kTileUnits;
   #pragma unroll
@@ -641,8 +651,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         const int sv = i % kStagesV;
         const int sb = i & 1;
         const int j = i >> 1;
-        if (!wait_bar(&bars->p_full[sb], j & 1, bars, p.err)) return false;
-        if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err)) return false;
+        if (!wait_bar(&bars->p_full[sb], j & 1, bars, p)) return false;
+        if (!wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p)) return false;
         tc_fence_after();
         const uint64_t vd = v_desc0 + sv * kTileUnits;
         // O_g += P_g(i) * V(i)[64g, 64g + 64): P_g is packed over columns
@@ -664,16 +674,13 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         if (!issue_pv(i)) { ok = false; break; }
         if (i + 2 < nt && !issue_qk(i + 2)) { ok = false; break; }
       }
-      if (!ok && any_mma) {
-        tc_commit_elect(&bars->drain);
-        mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
-      }
+      mma_issued = any_mma;
     } else if (warp == 3) {
       // ======================= cluster merge: K ring hand-off =======================
       // Once this CTA's last Q*K^T has completed no copy or MMA touches its K
       // ring again: tell the other splits they may write their rows into it.
       if (cmerge) {
-        const bool freed = wait_bar(&bars->kfree, 0, bars, p.err);
+        const bool freed = wait_bar(&bars->kfree, 0, bars, p);
         cluster_wait();
         cwaited = true;
         if (freed && lane == 0)
@@ -714,7 +721,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       const int sb = i & 1;
       const int c0 = (t_begin + i) * kBlockN + grp * 64;   // first key of this half
       const uint32_t t_s = t_row + sb * 128 + grp * 64;
-      if (ok) ok = wait_bar(&bars->s_full[sb], (i >> 1) & 1, bars, p.err);
+      if (ok) ok = wait_bar(&bars->s_full[sb], (i >> 1) & 1, bars, p);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       float s[64];
@@ -754,7 +761,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       // S(i) complete implies P*V(i-2) complete (issued before Q*K^T(i)), so
       // this parity wait on o_done[(i-1) & 1] cannot alias an older phase.
       if (warp_need && i > 0) {
-        if (ok) ok = wait_bar(&bars->o_done[(i - 1) & 1], ((i - 1) >> 1) & 1, bars, p.err);
+        if (ok) ok = wait_bar(&bars->o_done[(i - 1) & 1], ((i - 1) >> 1) & 1, bars, p);
         tc_fence_after();
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
@@ -772,7 +779,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       // rows of its own half.
       if (c0 + 64 > kv_end) {
         const int sv = i % kStagesV;
-        if (ok) ok = wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p.err);
+        if (ok) ok = wait_bar(&bars->v_full[sv], (i / kStagesV) & 1, bars, p);
         const int key = grp * 64 + (m & 63);
         if (ok && m < 64 && c0 + (m & 63) >= kv_end) {
           uint8_t* vrow = smem + kOffV + sv * kTileBytes + (key >> 3) * 1024 + (key & 7) * 128;
@@ -834,7 +841,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     grid_launch_dependents();
     // The last P*V completes after every other MMA of the CTA; P*V(nt-3) is
     // known complete, so the parity wait cannot alias an older phase.
-    if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p.err);
+    if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p);
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_after();
 
@@ -894,7 +901,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         fence_proxy_async_smem();   // the bulk copy reads through the async proxy
         named_bar_sync(2 + q, 64);  // this quadrant's warp of each group
         if (grp == 0 && lane == 0) {
-          if (wait_bar_cluster(&bars->go, 0, bars, p.err)) {
+          if (wait_bar_cluster(&bars->go, 0, bars, p)) {
             const int slot = (split < owner ? split : split - 1) * 2 + q / active;
             const uint32_t rbar = mapa_shared(smem_u32(&bars->ready), owner);
             bulk_copy_to_cluster(mapa_shared(sbase + kOffK + slot * kQuadBytes, owner), stage,
@@ -905,7 +912,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
           }
         }
       } else if (q * 32 < n_rows) {
-        const bool got = wait_bar_cluster(&bars->ready, 0, bars, p.err);
+        const bool got = wait_bar_cluster(&bars->ready, 0, bars, p);
         if (got && ok && row_ok) {
           const int j = q / active;
           const uint32_t rx = sbase + kOffK + j * kQuadBytes + lane * 512u;
@@ -976,9 +983,31 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   if (p.cluster && !cwaited) cluster_wait();
   // Every other split's `go` arrive has landed before this CTA's shared
   // memory goes away.
-  if (cmerge && threadIdx.x == 0) wait_bar_cluster(&bars->go, 0, bars, p.err);
+  if (cmerge && threadIdx.x == 0) wait_bar_cluster(&bars->go, 0, bars, p);
   tc_fence_before();
   __syncthreads();
+  // A CTA that unwound after a failed wait may still have MMAs in flight (the
+  // waits that would have seen them complete gave up): the MMA warp lets them
+  // finish before the tensor memory they write is freed. The abort flag is
+  // settled here (every thread has passed its last wait), so the branch is
+  // uniform over the CTA.
+  // Likewise the producers let their last tensor copies land (a ring that
+  // finished issuing before the abort was raised has not drained), so no copy
+  // writes into this CTA's shared memory after it exits.
+  if (*reinterpret_cast<volatile int*>(&bars->abort) != 0) {
+    if (warp == 1 && mma_issued) {
+      tc_commit_elect(&bars->drain);
+      mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
+    }
+    if (warp == 0) {
+      drain_ring(bars->k_full, kStagesK, issued, lane);
+      if (lane == 0) mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
+    } else if (warp == 2) {
+      drain_ring(bars->v_full, kStagesV, issued, lane);
+    }
+    tc_fence_before();
+    __syncthreads();
+  }
   if (warp == 3) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);

@@ -53,13 +53,17 @@ def test_status_strings_and_version(lib):
 
 
 def test_desc_struct_layout_matches_c():
-    # 12 int32 + float, then a pointer aligned to 8
-    assert ctypes.sizeof(zb.AttnDesc) == 64
+    # 12 int32 + float, a pointer aligned to 8, then the wait limit and the debug flags
+    assert ctypes.sizeof(zb.AttnDesc) == 72
     assert zb.AttnDesc.q_row_offsets.offset == 56
+    assert zb.AttnDesc.wait_limit_us.offset == 64
+    assert zb.AttnDesc.debug_flags.offset == 68
 
 
 @pytest.mark.parametrize("bad,status", [
     (dict(batch=0), 1),
+    (dict(wait_limit_us=-1), 1),
+    (dict(debug_flags=2), 1),
     (dict(n_q_heads=12, n_kv_heads=8), 1),
     (dict(dtype=7), 1),
     (dict(max_rows=0), 1),
