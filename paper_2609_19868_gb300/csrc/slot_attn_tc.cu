@@ -330,19 +330,28 @@ __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* 
   const bool paged = p.page_size > 0;
   const int ppt = paged ? kBlockN / p.page_size : 0;   // pages per tile
   const uint32_t page_bytes = paged ? static_cast<uint32_t>(p.page_size) * 256u : 0u;
+  // Lane l's page of tile i (-1 when the tile has no such page). The page ids
+  // of the next tile are read one tile ahead, before this tile's waits, so
+  // their latency hides behind the ring instead of delaying the copies.
+  auto page_of = [&](int i) -> int {
+    const int lp = (t_begin + i) * ppt + lane;
+    if (lane >= ppt || lp * p.page_size >= kv_end) return -1;
+    return p.page_table[static_cast<long long>(b) * p.max_pages + lp];
+  };
+  int page_next = (paged && i_begin < i_end) ? page_of(i_begin) : -1;
   for (int i = i_begin; i < i_end; ++i) {
     const int t = t_begin + i;
-    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p)) return false;
     int page = -1;
     uint32_t bytes = kTileBytes;
     if (paged) {
+      page = page_next;
+      if (i + 1 < i_end) page_next = page_of(i + 1);
+    }
+    if (t == t_stage && !wait_bar(&bars->staged, 0, bars, p)) return false;
+    if (paged) {
       const int lp = t * ppt + lane;
       const bool want = lane < ppt && lp * p.page_size < kv_end;
-      bool bad = false;
-      if (want) {
-        page = p.page_table[static_cast<long long>(b) * p.max_pages + lp];
-        bad = page < 0 || page >= p.n_pages;
-      }
+      const bool bad = want && (page < 0 || page >= p.n_pages);
       if (__any_sync(0xffffffffu, bad)) {
         if (lane == 0) set_abort(bars, p.err, ZARYA_DEVERR_PAGE_ID);
         return false;
@@ -430,10 +439,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   const int kvh = bh - b * p.Hkv;
 
   // ---- set-up that needs no input (overlaps the previous kernel's tail) ----
-  if (warp == 3) {
-    tmem_alloc(&bars->tmem_base, kTmemCols);
-    tmem_relinquish();
-  }
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&map_q);
     tma_prefetch_map(&map_k);
@@ -470,6 +475,10 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   // initialisation and be lost, and the producers' wait for it would run out.
   // No copy is in flight yet, so nothing holds a thread here.
   __syncthreads();
+  if (warp == 3) {
+    tmem_alloc(&bars->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
   // The producer warps load before the CTA-wide set-up barrier (a thread
   // with tensor copies in flight waits for them at a barrier): they arrive,
   // without waiting, on the set-up barrier the other ten warps wait on.
@@ -839,26 +848,30 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
     const long long unit = static_cast<long long>(bh) * p.m_tiles + mt;
     const int col0 = grp * 64;   // group g finishes columns [64g, 64g + 64)
     grid_launch_dependents();
+    // The cluster barrier's wait (needed before the merge's first remote
+    // access) is taken here, while the last P*V still runs.
+    if (p.cluster) {
+      cluster_wait();
+      cwaited = true;
+    }
     // The last P*V completes after every other MMA of the CTA; P*V(nt-3) is
     // known complete, so the parity wait cannot alias an older phase.
     if (ok) ok = wait_bar(&bars->o_done[(nt - 1) & 1], ((nt - 1) >> 1) & 1, bars, p);
     ok = __all_sync(0xffffffffu, ok);
     tc_fence_after();
 
-    // This CTA's result for its 64 columns of row m, normalised.
+    // This CTA's result for its 64 columns of row m, normalised: O_0's
+    // columns, then O_1's, one tensor-memory load (and wait) each.
     float o[64];
+    if (ok) {
+      tmem_ld_32x32b_x64(t_row + kTmemO + col0, o);
+      float vb[64];
+      tmem_ld_32x32b_x64(t_row + kTmemO + 128 + col0, vb);
 #pragma unroll
-    for (int ch = 0; ch < 2; ++ch) {
-      float va[32], vb[32];
-      if (ok) {
-        tmem_ld_32x32b_x32(t_row + kTmemO + col0 + ch * 32, va);
-        tmem_ld_32x32b_x32(t_row + kTmemO + 128 + col0 + ch * 32, vb);
-      } else {
+      for (int x = 0; x < 64; ++x) o[x] = wA * o[x] + wB * vb[x];
+    } else {
 #pragma unroll
-        for (int x = 0; x < 32; ++x) va[x] = vb[x] = 0.f;
-      }
-#pragma unroll
-      for (int x = 0; x < 32; ++x) o[ch * 32 + x] = wA * va[x] + wB * vb[x];
+      for (int x = 0; x < 64; ++x) o[x] = 0.f;
     }
     __nv_bfloat16* out_row = reinterpret_cast<__nv_bfloat16*>(p.out) +
                              (static_cast<long long>(row0 + r) * p.Hq + h) * kHeadDim + col0;
@@ -886,8 +899,6 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       const int q = wq;                                          // this warp's quadrant
       const int owner = q % active;
       const uint32_t sbase = smem_u32(smem);
-      cluster_wait();
-      cwaited = true;
       if (q * 32 < n_rows && owner != split) {
         const uint32_t stage = sbase + kOffV + q * kQuadBytes;
         const uint32_t stage_lse = sbase + kOffV + kRxLse + q * kQuadLseBytes;
