@@ -1252,6 +1252,78 @@ def run_mode_a(args):
     print(json.dumps(line), flush=True)
 
 
+def run_top_p(args):
+    """top_p truncation of the draft block's logits (Sec. 5.1 step 3, Table 2):
+    zarya_top_p in place over the decode block's 256 rows of the Qwen3
+    vocabulary (bf16). The call changes its input, so every call gets a fresh
+    copy of the logits, written just before it (as the LM head would leave
+    them, in L2); CUDA events bracket the top_p call alone. A draft pass over
+    the same logits is timed beside it for scale."""
+    import torch
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2609_19868_gb300 import build as zbuild
+
+    zbuild.build()
+    from paper_2609_19868_gb300 import _binding as zb
+    from paper_2609_19868_gb300 import session
+    from paper_2609_19868_gb300 import workloads as wl
+
+    zb.load()
+    zb.check_device_error()
+    name = args.workload if args.workload in SELECT_LABELS else "select_decode_small"
+    w = wl.make_sampling(name, device=dev)
+    T, top_p = args.temperature, args.top_p
+    sb = session.upload_sampling(w, dev, temperature=T)
+    src = sb.draft_logits.clone()
+    stream = torch.cuda.Stream(dev)
+    K, W = args.steps, args.warmup
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(K)]
+    with torch.cuda.stream(stream):
+        for i in range(W + K):
+            sb.draft_logits.copy_(src)
+            if i >= W:
+                evs[i - W][0].record(stream)
+            zb.top_p(sb.draft_logits, top_p, sb.draft_desc, stream=stream)
+            if i >= W:
+                evs[i - W][1].record(stream)
+    torch.cuda.synchronize()
+    assert zb.check_device_error(stream) == 0
+    ms = sorted(a.elapsed_time(b) for a, b in evs)
+    med = float(np.median(ms))
+    kept = int(torch.isfinite(sb.draft_logits.float()).sum().item())
+    with torch.cuda.stream(stream):
+        sb.draft_logits.copy_(src)
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        sb.draft(stream)
+        d0.record(stream)
+        for _ in range(K):
+            sb.draft(stream)
+        d1.record(stream)
+    torch.cuda.synchronize()
+    draft_ms = d0.elapsed_time(d1) / K
+    nbytes = w.rows * w.V * 2
+    line = {
+        "metric": "top_p calls/s (nucleus truncation of every row of a block's logits)",
+        "value": round(1e3 / med, 2), "unit": "calls/s", "n_gpus": 1, "steps": K, "warmup": W,
+        "ms_per_step": round(med, 5), "ms_per_step_min": round(ms[0], 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32 masses in 2^-40 fixed point (bf16 logits)",
+        "data": "synthetic (seeded N(0,2^2) logits with peaked tokens)",
+        "config": {"workload": SELECT_LABELS[name], "temperature": T, "top_p": top_p,
+                   "rows": w.rows, "kept_tokens": kept,
+                   "l2": "logits rewritten before every call (L2-warm, as after the LM head)"},
+        "draft_pass_ms": round(draft_ms, 5),
+        "ratio_to_draft_pass": round(med / draft_ms, 2),
+        "row_bytes_read_per_call": nbytes,
+        "gpu_launches": K,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def _oracle_select_rows(w, T, n_draft, n_verify, vtokens):
     """The sampling oracle over the first n_draft draft rows and n_verify
     verification rows (the per-row work dominates; the per-sequence rules are
@@ -1483,11 +1555,12 @@ def main():
                     help="each per_config entry's repeated regions last at least this long")
     ap.add_argument("--no-per-config", dest="per_config", action="store_false",
                     help="measure the chosen workload only")
-    ap.add_argument("--path", choices=["attention", "select", "reorder", "mode_a"],
+    ap.add_argument("--path", choices=["attention", "select", "reorder", "mode_a", "top_p"],
                     default="attention",
                     help="attention: the slot-decode layer step (stage + attention + commit); "
                          "select: slot selection + token acceptance over logits")
     ap.add_argument("--temperature", type=float, default=0.0)
+    ap.add_argument("--top-p", type=float, default=0.9)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--no-clocks", dest="clocks", action="store_false")
@@ -1495,11 +1568,18 @@ def main():
     if args.warmup < 3:
         args.warmup = 3
     if args.workload is None:
-        args.workload = "select_decode_small" if args.path == "select" else "serving_mix"
+        args.workload = ("select_decode_small" if args.path in ("select", "top_p")
+                         else "serving_mix")
     args.workload = WORKLOAD_ALIASES.get(args.workload, args.workload)
-    if args.path == "attention" and args.workload not in WORKLOAD_LABELS:
+    if args.path in ("attention",) and args.workload not in WORKLOAD_LABELS:
         ap.error(f"--workload {args.workload} is not an attention workload")
-    if args.path == "mode_a":
+    if args.path == "top_p":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable":
+                              "the top_p path is measured against a draft pass only"}), flush=True)
+        else:
+            run_top_p(args)
+    elif args.path == "mode_a":
         if args.impl == "reference":
             print(json.dumps({"impl": "reference", "unavailable":
                               "the Mode A path is measured against its roofline only"}), flush=True)

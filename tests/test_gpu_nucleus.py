@@ -2,8 +2,8 @@
 row on fp32 and bf16 rows (heavy ties in bf16), several temperatures and top_p
 values, rows of no sequence, and draws taken after the truncation. The GPU
 sums masses in fixed point from fp32 exponentials, so a kept set may differ
-from the exact one only where the mass at a boundary is within 1e-5 of
-top_p; every difference is checked to be such a case."""
+from the exact one only in one logit value whose boundary mass is within
+2e-6 of top_p; every difference is checked to be such a case."""
 import numpy as np
 import pytest
 import torch
@@ -51,18 +51,29 @@ def _run(zb, x, dtype, row_offsets, T, top_p, max_slots=1):
     return logits, ro, d
 
 
+# The kernel's masses are fp32 exponentials of fp32 arguments summed in 2^-40
+# fixed point: relative to the exact masses they are off by less than 1e-6 (the
+# argument's rounding dominates), so the boundary value x* can come out one
+# distinct value off only when the exact cumulative mass at that boundary lies
+# within this margin of top_p.
+BOUNDARY_MARGIN = 2e-6
+
+
 def _kept_ok(x_row, gpu_kept, T, top_p):
     """The GPU's kept set (over the finite logits) equals the oracle's, or
-    differs only at boundaries whose exact mass is within 1e-5 of top_p."""
+    differs in one distinct logit value whose boundary mass (the exact mass
+    of the tokens at or above it, or strictly above it) lies within
+    BOUNDARY_MARGIN of top_p."""
     fin = np.isfinite(x_row)
     want = nuc.kept_mask(x_row, T, top_p)
     if np.array_equal(gpu_kept[fin], want[fin]):
         return True
+    diff = np.unique(x_row[fin & (gpu_kept != want)])
+    if len(diff) != 1:
+        return False
     p = nuc._probs(x_row, T)
-    for v in np.unique(x_row[fin & (gpu_kept != want)]):
-        if min(abs(p[x_row >= v].sum() - top_p), abs(p[x_row > v].sum() - top_p)) > 1e-5:
-            return False
-    return True
+    v = diff[0]
+    return min(abs(p[x_row >= v].sum() - top_p), abs(p[x_row > v].sum() - top_p)) <= BOUNDARY_MARGIN
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
