@@ -89,6 +89,7 @@ zarya_status check_attn_support(const zarya_attn_desc* d) {
 
 struct Plan {
   int g, m_tiles, splits;
+  int pair;   // one CTA per pair of M-tiles (grid.x = pairs)
   long long units;
   size_t off_lse, off_cnt, bytes;
 };
@@ -107,6 +108,16 @@ Plan plan_tc(const zarya_attn_desc* d, int sms) {
   p.units = static_cast<long long>(d->batch) * d->n_kv_heads * p.m_tiles;
   const long long kv_max = d->max_kv_len > 0 ? d->max_kv_len : d->cache_capacity;
   const int tiles = static_cast<int>((kv_max + kBlockN - 1) / kBlockN);
+  // Paged caches cost one tensor copy per page per tile; serving two M-tiles
+  // of a (sequence, KV head) from each tile halves the copies per unit of
+  // work. Taken when the pairs alone fill the GPU (no key split needed).
+  const long long pairs = (p.m_tiles + 1) / 2;
+  if (d->page_size > 0 && d->kv_splits == 0 && p.m_tiles >= 2 &&
+      static_cast<long long>(d->batch) * d->n_kv_heads * pairs >= sms) {
+    p.pair = 1;
+    p.splits = 1;
+    return p;
+  }
   int splits = 1;
   if (d->kv_splits > 0) {
     splits = d->kv_splits < tiles ? d->kv_splits : tiles;
@@ -350,6 +361,7 @@ zarya_status slot_attn_impl(const void* q, const void* k_new, const void* v_new,
   p.m_tiles = plan.m_tiles;
   p.splits = plan.splits;
   p.cluster = (plan.splits > 1 && plan.splits <= kMaxClusterSplits) ? 1 : 0;
+  p.pair = plan.pair;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.wait_ns = desc->wait_limit_us > 0 ? static_cast<uint64_t>(desc->wait_limit_us) * 1000ull
                                        : 2000000000ull;

@@ -37,6 +37,7 @@ struct TcParams {
   int page_size, max_pages, n_pages;
   int m_tiles, splits;
   int cluster;        // 1: the splits of a tile form a cluster and merge through DSMEM
+  int pair;           // 1: one CTA per pair of M-tiles (paged caches, no key split)
   float scale_log2;   // softmax scale * log2(e)
   uint64_t wait_ns;   // bound on every pipeline wait (global-timer nanoseconds)
   int debug_stall;    // 1: the MMA warp first waits on a barrier nothing completes

@@ -114,19 +114,36 @@ __device__ __forceinline__ void named_bar_arrive(int id, int n) {
   asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 
+// Named barrier that also ANDs a flag over its n threads (every participant
+// arrives whatever its flag, so the group leaves together).
+__device__ __forceinline__ bool named_bar_and(int id, int n, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %3, 0;\n\t"
+      "bar.red.and.pred po, %1, %2, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"(id), "r"(n), "r"(v ? 1u : 0u)
+      : "memory");
+  return r != 0;
+}
+
 // Named barriers (barrier 0 is __syncthreads): 1 joins the 256 softmax
 // threads, 2-5 one quadrant's warp of each softmax group, 7 publishes the
 // entry set-up to the other ten warps.
 constexpr int kBarSoftmax = 1;
 constexpr int kBarSetup = 7;
 
-__device__ __forceinline__ void set_abort(Bars* bars, int* err, int code) {
+template <class BarsT>
+__device__ __forceinline__ void set_abort(BarsT* bars, int* err, int code) {
   record_error(err, code);
   *reinterpret_cast<volatile int*>(&bars->abort) = 1;
 }
 
 // Bounded wait (p.wait_ns of global time) for a phase of a barrier of this CTA.
-__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, Bars* bars,
+template <class BarsT>
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, BarsT* bars,
                                          const TcParams& p) {
   if (mbar_wait(bar, parity, p.wait_ns, &bars->abort)) return true;
   set_abort(bars, p.err, ZARYA_DEVERR_TIMEOUT);
@@ -322,9 +339,10 @@ struct GroupStager {
 // [i_begin, i_end) of this CTA's range, `issued` counting the tiles whose
 // copies are in flight. Returns false (the CTA aborts) on a bad page id or a
 // timed-out wait.
+template <class BarsT>
 __device__ __forceinline__ bool produce_range(const CUtensorMap* map, uint64_t* full,
                                               uint64_t* empty, int stages, uint32_t ring,
-                                              const TcParams& p, Bars* bars, int b, int kvh,
+                                              const TcParams& p, BarsT* bars, int b, int kvh,
                                               int t_begin, int i_begin, int i_end, int kv_end,
                                               int lane, int t_stage, int& issued) {
   const bool paged = p.page_size > 0;
@@ -1025,6 +1043,466 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
   }
 }
 
+// ---------------------------------------------------------------------------
+// Paired M-tiles (paged caches). One CTA serves two M-tiles A = 2*pair and
+// B = 2*pair + 1 of one (sequence, KV head) from every K/V tile it loads, so
+// the tensor copies per unit of work halve; with 16-token pages the per-copy
+// cost, not the tensor pipe, otherwise sets the pace.
+//
+// The work is a sequence of jobs, one per (tile, M-tile): with B present,
+// job j is M-tile j & 1 of tile j >> 1; without B (a sequence too short for
+// it), job j is tile j of A. Job j's S goes to TMEM columns [128 (j & 1), +128)
+// (S_A / S_B, or S double-buffered for A alone); each M-tile has one O
+// accumulator, O_A [256, 384) and O_B [384, 512). The MMA order is the single
+// M-tile kernel's with jobs for tiles: Q*K^T(0), Q*K^T(1), then P*V(j),
+// Q*K^T(j + 2); one thread's MMAs complete in order, so Q*K^T(j + 2) cannot
+// overwrite P(j) before P*V(j) has read it, and a completed Q*K^T(j) implies
+// P*V(j - 2) has completed.
+//
+// Both softmax groups work on every job: group g takes keys [64g, 64g + 64)
+// of the tile, but the two share the row maximum (each leaves its half's
+// maximum in a spare TMEM column of its half, the quadrant's two warps meet
+// at a named barrier, and each reads the other's), so one O per M-tile
+// suffices: each group rescales and finishes columns [64g, 64g + 64) of it,
+// and the groups' row sums add at the end. The key range is not split (one
+// CTA per pair).
+constexpr int kPairStagesK = 3;
+constexpr int kPairStagesV = 2;
+constexpr uint32_t kPOffQ = 0;                                   // Q_A, then Q_B
+constexpr uint32_t kPOffK = 2 * kTileBytes;
+constexpr uint32_t kPOffV = kPOffK + kPairStagesK * kTileBytes;
+constexpr uint32_t kPOffBar = kPOffV + kPairStagesV * kTileBytes;
+
+struct PairBars {
+  uint64_t q_full;
+  uint64_t k_full[kPairStagesK];
+  uint64_t k_empty[kPairStagesK];
+  uint64_t v_full[kPairStagesV];
+  uint64_t v_empty[kPairStagesV];
+  uint64_t s_full[2];   // [j & 1]: Q*K^T(j) has completed (phase j >> 1)
+  uint64_t p_full[2];   // [j & 1]: P(j) is written (8 warps, phase j >> 1)
+  uint64_t o_done[2];   // [j & 1]: P*V(j) has completed (phase j >> 1)
+  uint64_t drain;
+  uint64_t staged;
+  uint64_t stage_issued;
+  uint64_t stall;
+  uint32_t tmem_base;
+  int abort;
+};
+
+constexpr uint32_t kPairSmemBytes = kPOffBar + ((sizeof(PairBars) + 127) / 128) * 128 + 1024;
+static_assert(kPairSmemBytes <= 232448, "shared memory budget (paired M-tiles)");
+
+// Row maximum of 64 scores.
+__device__ __forceinline__ float max64(const float (&s)[64]) {
+  float m8[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) m8[k] = s[k];
+#pragma unroll
+  for (int x = 8; x < 64; x += 8)
+#pragma unroll
+    for (int k = 0; k < 8; ++k) m8[k] = fmaxf(m8[k], s[x + k]);
+  return fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
+                      const __grid_constant__ CUtensorMap map_k,
+                      const __grid_constant__ CUtensorMap map_v, const TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  PairBars* bars = reinterpret_cast<PairBars*>(smem + kPOffBar);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int pair = blockIdx.x;
+  const int bh = blockIdx.z;
+  const int b = bh / p.Hkv;
+  const int kvh = bh - b * p.Hkv;
+
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&map_q);
+    tma_prefetch_map(&map_k);
+    tma_prefetch_map(&map_v);
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->q_full, 1);
+    for (int s = 0; s < kPairStagesK; ++s) {
+      mbar_init(&bars->k_full[s], 1);
+      mbar_init(&bars->k_empty[s], 1);
+    }
+    for (int s = 0; s < kPairStagesV; ++s) {
+      mbar_init(&bars->v_full[s], 1);
+      mbar_init(&bars->v_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bars->s_full[s], 1);
+      mbar_init(&bars->p_full[s], kSoftmaxWarps);
+      mbar_init(&bars->o_done[s], 1);
+    }
+    mbar_init(&bars->drain, 1);
+    mbar_init(&bars->staged, kSoftmaxWarps);
+    mbar_init(&bars->stage_issued, kSoftmaxWarps);
+    mbar_init(&bars->stall, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  // every barrier is initialised before any thread touches one
+  __syncthreads();
+  if (warp == 3) {
+    tmem_alloc(&bars->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == 0 || warp == 2) named_bar_arrive(kBarSetup, kThreads);
+  // Inputs may be written by the kernel launched before this one.
+  grid_dependency_wait();
+
+  // ---- per-sequence geometry (uniform over the CTA) ----
+  const int P = p.cache_lens[b];
+  const long long R64 = static_cast<long long>(p.n_slots[b]) * p.slot_len[b];
+  const int R = R64 > p.max_rows ? p.max_rows + 1 : static_cast<int>(R64);
+  const int mode = p.mask_mode[b];
+  const int row0 = p.q_row_offsets[b];
+  const int row_end = p.q_row_offsets[b + 1];
+  int code = 0;
+  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL &&
+      mode != ZARYA_MASK_SLOT_INDEPENDENT)
+    code = ZARYA_DEVERR_MASK_MODE;
+  else if (p.n_slots[b] < 1 || p.slot_len[b] < 1 || R > p.max_rows || row_end - row0 != R ||
+           row0 < 0 || row_end > p.total_rows)
+    code = ZARYA_DEVERR_ROWS;
+  else if (P < 0 || static_cast<long long>(P) + R > p.capacity) code = ZARYA_DEVERR_CAPACITY;
+  const int rows_per_tile = kBlockM / p.g;
+  const int r0A = 2 * pair * rows_per_tile;
+  const int r0B = r0A + rows_per_tile;
+  const bool hasB = r0B < R;
+  const int r_hi = min(r0A + 2 * rows_per_tile, R) - 1;   // last block row of the pair
+  const int kv_end = (mode == ZARYA_MASK_BIDIR_BLOCK) ? P + R : P + r_hi + 1;
+  const int nt = (code != 0 || kv_end <= 0) ? 1 : (kv_end + kBlockN - 1) / kBlockN;
+  const int njobs = hasB ? 2 * nt : nt;
+  const int jshift = hasB ? 1 : 0;   // tile of job j = j >> jshift
+  int st_lo = 0, st_hi = 0;   // staged attention: block rows read, relative to P
+  if (p.k_new != nullptr && code == 0) st_hi = kv_end - P;
+
+  const bool works = code == 0 && r0A < R;
+  const int t_stage = st_hi > st_lo ? P / kBlockN : -1;
+  int issued = 0;
+  const bool stage_here = works && st_hi > st_lo;
+  GroupStager stg;
+  if (warp >= 4 && stage_here) {
+    stg.load(p, b, kvh, row0, P, st_lo, st_hi, threadIdx.x - 128, 0);
+    __syncwarp();
+    if (lane == 0) mbar_arrive_relaxed(&bars->stage_issued);
+  }
+  if (warp == 0 && works && lane == 0) {
+    // Q of both M-tiles (B's rows past R_b are never stored)
+    mbar_arrive_expect_tx(&bars->q_full, (hasB ? 2u : 1u) * kTileBytes);
+    const uint32_t dq = smem_u32(smem + kPOffQ);
+    tma_load_3d(dq, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0A);
+    tma_load_3d(dq + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0A);
+    if (hasB) {
+      tma_load_3d(dq + kTileBytes, &map_q, &bars->q_full, 0, kvh * p.g, row0 + r0B);
+      tma_load_3d(dq + kTileBytes + kHalfBytes, &map_q, &bars->q_full, 64, kvh * p.g, row0 + r0B);
+    }
+  }
+  if ((warp == 0 || warp == 2) && works && stage_here) {
+    // a timeout sets the abort flag; the ring loop below then returns early
+    if (lane == 0) wait_bar(&bars->stage_issued, 0, bars, p);
+    __syncwarp();
+  }
+  if (warp != 0 && warp != 2) {
+    tc_fence_before();
+    named_bar_sync(kBarSetup, kThreads);
+    tc_fence_after();
+  }
+  const uint32_t tmem = (warp != 0 && warp != 2) ? bars->tmem_base : 0u;
+  bool mma_issued = false;
+  if (!works) {
+    if (code != 0 && pair == 0 && threadIdx.x == 0) record_error(p.err, code);
+    grid_launch_dependents();
+    if (warp == 3) tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
+
+  if (warp < 4) {
+    if (warp == 0) {
+      if (!produce_range(&map_k, bars->k_full, bars->k_empty, kPairStagesK,
+                         smem_u32(smem + kPOffK), p, bars, b, kvh, 0, 0, nt, kv_end, lane, t_stage,
+                         issued))
+        drain_ring(bars->k_full, kPairStagesK, issued, lane);
+      if (lane == 0 && *reinterpret_cast<volatile int*>(&bars->abort) != 0)
+        mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
+    } else if (warp == 2) {
+      if (!produce_range(&map_v, bars->v_full, bars->v_empty, kPairStagesV,
+                         smem_u32(smem + kPOffV), p, bars, b, kvh, 0, 0, nt, kv_end, lane, t_stage,
+                         issued))
+        drain_ring(bars->v_full, kPairStagesV, issued, lane);
+    } else if (warp == 1) {
+      // ======================= MMA issuer (one elected lane) =======================
+      bool ok = true;
+      if (p.debug_stall) ok = wait_bar(&bars->stall, 0, bars, p);
+      if (ok) ok = wait_bar(&bars->q_full, 0, bars, p);
+      bool any_mma = false;
+      tc_fence_after();
+      const uint32_t q0 = smem_u32(smem + kPOffQ);
+      const uint64_t k_desc0 = sdesc_sw128(smem_u32(smem + kPOffK), 16, 1024);
+      const uint64_t v_desc0 = sdesc_sw128(smem_u32(smem + kPOffV), kHalfBytes, 1024);
+      constexpr uint64_t kTileUnits = kTileBytes >> 4, kHalfUnits = kHalfBytes >> 4;
+      // A tile's first job waits for its K (V) tile; its last job releases it.
+      auto first_of_tile = [&](int j) { return !hasB || (j & 1) == 0; };
+      auto last_of_tile = [&](int j) { return !hasB || (j & 1) == 1; };
+      auto issue_qk = [&](int j) -> bool {
+        const int i = j >> jshift;
+        const int s = i % kPairStagesK;
+        const int t = hasB ? (j & 1) : 0;
+        if (first_of_tile(j)) {
+          if (!wait_bar(&bars->k_full[s], (i / kPairStagesK) & 1, bars, p)) return false;
+          tc_fence_after();
+        }
+        const uint32_t qt = q0 + t * kTileBytes;
+        const uint64_t qd0 = sdesc_sw128(qt, 16, 1024);
+        const uint64_t qd1 = sdesc_sw128(qt + kHalfBytes, 16, 1024);
+        const uint64_t kd = k_desc0 + s * kTileUnits;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t step = (kk >> 2) * kHalfUnits + (kk & 3) * 2;
+          tc_mma_ss_elect(tmem + (j & 1) * 128, (kk < 4 ? qd0 : qd1) + (kk & 3) * 2, kd + step,
+                          kIdescQK, kk > 0 ? 1u : 0u);
+        }
+        any_mma = true;
+        tc_commit_elect(&bars->s_full[j & 1]);
+        if (last_of_tile(j)) tc_commit_elect(&bars->k_empty[s]);
+        return true;
+      };
+      // O_t += P(j) V: group g's P is packed over columns [64g, 64g + 32) of S(j)
+      auto issue_pv = [&](int j) -> bool {
+        const int i = j >> jshift;
+        const int sv = i % kPairStagesV;
+        const int t = hasB ? (j & 1) : 0;
+        if (!wait_bar(&bars->p_full[j & 1], (j >> 1) & 1, bars, p)) return false;
+        if (first_of_tile(j)) {
+          if (!wait_bar(&bars->v_full[sv], (i / kPairStagesV) & 1, bars, p)) return false;
+        }
+        tc_fence_after();
+        const uint64_t vd = v_desc0 + sv * kTileUnits;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          tc_mma_ts_elect(tmem + kTmemO + t * 128, tmem + (j & 1) * 128 + (c >> 2) * 64 + (c & 3) * 8,
+                          vd + c * 128, kIdescPV, (i > 0 || c > 0) ? 1u : 0u);
+        any_mma = true;
+        tc_commit_elect(&bars->o_done[j & 1]);
+        if (last_of_tile(j)) tc_commit_elect(&bars->v_empty[sv]);
+        return true;
+      };
+      if (ok) ok = issue_qk(0);
+      if (ok && njobs > 1) ok = issue_qk(1);
+      for (int j = 0; j < njobs && ok; ++j) {
+        if (!issue_pv(j)) { ok = false; break; }
+        if (j + 2 < njobs && !issue_qk(j + 2)) { ok = false; break; }
+      }
+      mma_issued = any_mma;
+    }
+  } else {
+    // ======================= softmax + epilogue =======================
+    if (stage_here) {
+      stg.finish(p, b, kvh, row0, P, st_lo, st_hi, threadIdx.x - 128);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->staged);
+    }
+    const int grp = (warp - 4) >> 2;
+    const int wq = warp & 3;
+    const int m = wq * 32 + lane;   // packed row = TMEM lane (of both M-tiles)
+    const int h = kvh * p.g + (m - (m / p.g) * p.g);
+    // this lane's block row of M-tile t is r0A + t * rows_per_tile + mrow
+    const int mrow = m / p.g;
+    const int L = p.slot_len[b];
+    auto row_of = [&](int t) { return r0A + t * rows_per_tile + mrow; };
+    auto row_valid = [&](int t) { return row_of(t) < R && (t == 0 || hasB); };
+    const uint32_t t_row = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+    const float sl2 = p.scale_log2;
+    float m_runA = -INFINITY, m_runB = -INFINITY;
+    float l_runA = 0.f, l_runB = 0.f;
+    bool ok = true;
+    auto mask64 = [&](float (&s)[64], int c0, int limit, int hide_hi) {
+      if (c0 + 64 > limit) {
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+          if (c0 + x >= limit) s[x] = -INFINITY;
+      }
+      if (hide_hi > P && c0 < hide_hi && c0 + 64 > P) {
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+          if (c0 + x >= P && c0 + x < hide_hi) s[x] = -INFINITY;
+      }
+    };
+    for (int j = 0; j < njobs; ++j) {
+      const int i = j >> jshift;
+      const int t = hasB ? (j & 1) : 0;
+      const int rt = row_of(t);
+      const bool okt = row_valid(t);
+      const int limit = !okt ? kv_end : (mode == ZARYA_MASK_BIDIR_BLOCK ? P + R : P + rt + 1);
+      const int hide_hi = (okt && mode == ZARYA_MASK_SLOT_INDEPENDENT) ? P + (rt / L) * L : P;
+      const uint32_t t_s = t_row + (j & 1) * 128;
+      const uint32_t t_o = t_row + kTmemO + t * 128 + grp * 64;
+      const int c_tile = i * kBlockN;
+      const int c0 = c_tile + grp * 64;   // this group's keys
+      if (ok) ok = wait_bar(&bars->s_full[j & 1], (j >> 1) & 1, bars, p);
+      ok = __all_sync(0xffffffffu, ok);
+      // This group's scores and their row maximum, which it leaves in column
+      // 32 of its half of S (a column that neither P nor P*V uses).
+      float s[64];
+      float mx = -INFINITY;
+      if (ok) {
+        tc_fence_after();
+        tmem_ld_32x32b_x64(t_s + grp * 64, s);
+        mask64(s, c0, limit, hide_hi);
+        mx = max64(s);
+        tmem_st_32x32b_x1(t_s + grp * 64 + 32, mx);
+        tc_fence_before();
+      }
+      // Both warps of the quadrant arrive here every job and leave together,
+      // going on only if both got their S; then each reads the other's maximum.
+      if (!named_bar_and(2 + wq, 64, ok)) { ok = false; break; }
+      tc_fence_after();
+      mx = fmaxf(mx, tmem_ld_32x32b_x1(t_s + (1 - grp) * 64 + 32));
+      float m_run = t ? m_runB : m_runA;
+      float l_run = t ? l_runB : l_runA;
+      const float m_new = fmaxf(m_run, mx * sl2);
+      const bool need = m_new > m_run + 8.0f;
+      const bool warp_need = __any_sync(0xffffffffu, need);
+      float alpha = 1.f;
+      if (warp_need) {
+        alpha = (m_run == -INFINITY) ? 0.f : fast_exp2(m_run - m_new);
+        m_run = m_new;
+        l_run *= alpha;
+      }
+      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
+      // Rescaling this group's half of O_t must wait for the last P*V that
+      // wrote O_t: job j - 2 with B present, j - 1 without (the S of job j
+      // completing implies P*V(j - 2) has completed, so neither parity wait
+      // can alias an older phase).
+      if (warp_need && i > 0) {
+        const int jp = hasB ? j - 2 : j - 1;
+        if (ok) ok = wait_bar(&bars->o_done[jp & 1], (jp >> 1) & 1, bars, p);
+        tc_fence_after();
+#pragma unroll
+        for (int ch = 0; ch < 2; ++ch) {
+          float v[32];
+          const uint32_t a = t_o + ch * 32;
+          tmem_ld_32x32b_x32(a, v);
+#pragma unroll
+          for (int x = 0; x < 32; ++x) v[x] *= alpha;
+          tmem_st_32x32b_x32(a, v);
+        }
+      }
+      // Keys at or past kv_end in the last tile: their V rows must be exact
+      // zeros before the tile's first P*V reads them; each group clears the
+      // rows of its half.
+      if ((!hasB || t == 0) && c0 + 64 > kv_end) {
+        const int sv = i % kPairStagesV;
+        if (ok) ok = wait_bar(&bars->v_full[sv], (i / kPairStagesV) & 1, bars, p);
+        const int key = grp * 64 + (m & 63);
+        if (ok && m < 64 && c0 + (m & 63) >= kv_end) {
+          uint8_t* vrow = smem + kPOffV + sv * kTileBytes + (key >> 3) * 1024 + (key & 7) * 128;
+          const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+          for (int x = 0; x < 8; ++x) {
+            reinterpret_cast<uint4*>(vrow)[x] = z;
+            reinterpret_cast<uint4*>(vrow + kHalfBytes)[x] = z;
+          }
+        }
+        fence_proxy_async_smem();
+      }
+      // P = 2^(s * scale * log2 e - m) for this group's keys, packed bf16
+      // pairs over the first 32 columns of its half of S.
+      float pk[32];
+      float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
+#pragma unroll
+      for (int x = 0; x < 32; x += 2) {
+        const int c = 2 * x;
+        const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
+        const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
+        const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
+        const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
+        rs0 += e0;
+        rs1 += e1;
+        rs2 += e2;
+        rs3 += e3;
+        pk[x] = __uint_as_float(pack_bf16(e0, e1));
+        pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
+      }
+      tmem_st_32x32b_x32(t_s + grp * 64, pk);
+      l_run += (rs0 + rs1) + (rs2 + rs3);
+      if (t) {
+        m_runB = m_run;
+        l_runB = l_run;
+      } else {
+        m_runA = m_run;
+        l_runA = l_run;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->p_full[j & 1]);
+    }
+
+    // ---- epilogue: the groups' row sums add (both used the same maxima);
+    // the Q buffer (read by no MMA any more) carries them ----
+    float* xch = reinterpret_cast<float*>(smem + kPOffQ);
+    xch[(grp * 2 + 0) * 128 + m] = l_runA;
+    xch[(grp * 2 + 1) * 128 + m] = l_runB;
+    named_bar_sync(kBarSoftmax, 256);
+    const float l_totA = xch[m] + xch[2 * 128 + m];
+    const float l_totB = xch[128 + m] + xch[3 * 128 + m];
+    grid_launch_dependents();
+    // P*V(njobs - 1) completes after every other MMA of the CTA
+    if (ok) ok = wait_bar(&bars->o_done[(njobs - 1) & 1], ((njobs - 1) >> 1) & 1, bars, p);
+    ok = __all_sync(0xffffffffu, ok);
+    tc_fence_after();
+#pragma unroll
+    for (int t = 0; t < 2; ++t) {
+      if (ok && row_valid(t)) {
+        const float l_tot = t ? l_totB : l_totA;
+        const float inv = (l_tot > 0.f) ? 1.f / l_tot : 0.f;
+        float o[64];
+        tmem_ld_32x32b_x64(t_row + kTmemO + t * 128 + grp * 64, o);
+        uint4* d4 = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) +
+                                             (static_cast<long long>(row0 + row_of(t)) * p.Hq +
+                                              h) * kHeadDim + grp * 64);
+#pragma unroll
+        for (int x = 0; x < 8; ++x)
+          d4[x] = make_uint4(pack_bf16(o[8 * x + 0] * inv, o[8 * x + 1] * inv),
+                             pack_bf16(o[8 * x + 2] * inv, o[8 * x + 3] * inv),
+                             pack_bf16(o[8 * x + 4] * inv, o[8 * x + 5] * inv),
+                             pack_bf16(o[8 * x + 6] * inv, o[8 * x + 7] * inv));
+      }
+    }
+  }
+
+  // ---- teardown (as the single-tile kernel's) ----
+  tc_fence_before();
+  __syncthreads();
+  if (*reinterpret_cast<volatile int*>(&bars->abort) != 0) {
+    if (warp == 1 && mma_issued) {
+      tc_commit_elect(&bars->drain);
+      mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
+    }
+    if (warp == 0) {
+      drain_ring(bars->k_full, kPairStagesK, issued, lane);
+      if (lane == 0) mbar_wait(&bars->q_full, 0, kDrainNs, nullptr);
+    } else if (warp == 2) {
+      drain_ring(bars->v_full, kPairStagesV, issued, lane);
+    }
+    tc_fence_before();
+    __syncthreads();
+  }
+  if (warp == 3) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
 }  // namespace
 
 size_t tc_smem_bytes() { return kSmemBytes; }
@@ -1039,14 +1517,17 @@ cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map
   if (configured_device != dev) {
     e = cudaFuncSetAttribute(slot_attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(kSmemBytes));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(slot_attn_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(kPairSmemBytes));
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
   cudaLaunchConfig_t cfg{};
   cudaLaunchAttribute attr[2]{};
-  cfg.gridDim = dim3(p.m_tiles, p.splits, p.B * p.Hkv);
+  cfg.gridDim = dim3(p.pair ? (p.m_tiles + 1) / 2 : p.m_tiles, p.splits, p.B * p.Hkv);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = p.pair ? kPairSmemBytes : kSmemBytes;
   cfg.stream = stream;
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
@@ -1059,6 +1540,7 @@ cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map
     cfg.numAttrs = 2;
   }
   cfg.attrs = attr;
+  if (p.pair) return cudaLaunchKernelEx(&cfg, slot_attn_pair_kernel, map_q, map_k, map_v, p);
   return cudaLaunchKernelEx(&cfg, slot_attn_tc_kernel, map_q, map_k, map_v, p);
 }
 
