@@ -89,12 +89,13 @@ def algorithmic_counts(w):
                 commit_bytes=int(2 * 2 * w.accept_len.astype(np.int64).sum() * row))
 
 
-def recorded_traffic(workload: str):
+def recorded_traffic(workload: str, kernel: str = "slot_attn_tc_kernel"):
     """DRAM bytes (read + write) of one attention launch from the committed ncu
-    summary, if it was taken on the current kernel sources; else None."""
+    summary (profiles/<kernel>_<workload>.json), if it was taken on the current
+    kernel sources; else None."""
     import hashlib
 
-    path = os.path.join(ROOT, "profiles", f"slot_attn_tc_{workload}.json")
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.json")
     try:
         with open(path) as f:
             rec = json.load(f)
@@ -296,7 +297,8 @@ def per_sequence_roofline(w, hbm_peak, tf_peak):
     return ideal, hbm_part, ideal - hbm_part, batch_wide
 
 
-def roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src, traffic):
+def roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src, traffic,
+                          kernel=None):
     """The attention launch against the per-sequence roofline of its batch.
 
     `bound` names the resource that bounds most of the ideal time. When every
@@ -329,7 +331,8 @@ def roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src, traff
              "frac_of_batch_wide_bound": round(batch_wide / t, 4),
              "intensity_flop_per_byte": round(counts["flops"] / counts["attn_bytes"], 1),
              "ridge_flop_per_byte": round(tf_peak * 1e12 / (hbm_peak * 1e9), 1),
-             "kernel": "slot_attn_tc_kernel" if w.dtype == "bf16" else "slot_attn_f32_kernel"}
+             "kernel": kernel or ("slot_attn_tc_kernel" if w.dtype == "bf16"
+                                  else "slot_attn_f32_kernel")}
     if mixed:
         entry["peak_measured"] = peak_meas
     if w.dtype != "bf16":
@@ -417,6 +420,7 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
         for _ in range(n_rot - 1):
             kc, vc = base.k_cache.clone(), base.v_cache.clone()
             rots.append(session.upload(w, dev, caches=(kc, vc)))
+    kernel = zb.slot_attn_kernel(base.desc)   # the kernel the plan launches
     # The commit writes the advanced lengths into a second array (the
     # ping-pong a decoding loop would use), so every step starts from the same
     # prefix lengths: a stationary workload with no copy between steps.
@@ -606,7 +610,7 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
         "h2d": int(h2d),
         "d2h": int(d2h),
         "roofline": roofline_per_sequence(w, counts, attn_ms, hbm_peak, tf_peak, peak_src,
-                                          recorded_traffic(entry)),
+                                          recorded_traffic(entry, kernel), kernel),
         "hbm_gbs": counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9,
         "tflops": counts["flops"] / (attn_ms * 1e-3) / 1e12,
         "steps_per_s": replica_throughput(K, world, step_ms * K),

@@ -139,6 +139,17 @@ typedef struct {
 size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc);
 
 /*
+ * Name of the kernel zarya_slot_attn launches for `desc` on the current
+ * device (for profilers and reports): "slot_attn_tc_kernel" (one M-tile of
+ * 128 packed rows per CTA, key range split across CTAs where that pays),
+ * "slot_attn_pair_kernel" (paged caches whose M-tile pairs fill the GPU: two
+ * M-tiles per CTA sharing every K/V tile), "slot_attn_f32_kernel" (fp32), or
+ * "none" for a descriptor zarya_slot_attn would reject. A static string; no
+ * device work.
+ */
+const char* zarya_slot_attn_kernel(const zarya_attn_desc* desc);
+
+/*
  * Slot attention (Sec. 5.2 steps 3 and 6): for every sequence b, query head
  * h and block row r < R_b,
  *   out[q_row_offsets[b] + r, h, :] =

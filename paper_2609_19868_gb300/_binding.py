@@ -93,6 +93,8 @@ def load() -> ctypes.CDLL:
     dp = ctypes.POINTER(AttnDesc)
     lib.zarya_slot_attn_workspace_size.argtypes = [dp]
     lib.zarya_slot_attn_workspace_size.restype = sz
+    lib.zarya_slot_attn_kernel.argtypes = [dp]
+    lib.zarya_slot_attn_kernel.restype = ctypes.c_char_p
     lib.zarya_slot_attn.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, dp, vp]
     lib.zarya_slot_attn.restype = ctypes.c_int
     lib.zarya_slot_attn_staged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
@@ -192,6 +194,11 @@ def make_desc(*, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int, dty
     d.q_row_offsets = q_row_offsets.data_ptr()
     d._keep = q_row_offsets  # keep the offsets alive as long as the descriptor
     return d
+
+
+def slot_attn_kernel(desc: AttnDesc) -> str:
+    """``zarya_slot_attn_kernel``: the kernel the plan for ``desc`` launches."""
+    return load().zarya_slot_attn_kernel(ctypes.byref(desc)).decode()
 
 
 def workspace_size(desc: AttnDesc) -> int:

@@ -209,6 +209,12 @@ using namespace zarya;
 
 extern "C" {
 
+const char* zarya_slot_attn_kernel(const zarya_attn_desc* desc) {
+  if (check_desc(desc) != ZARYA_OK || check_attn_support(desc) != ZARYA_OK) return "none";
+  if (desc->dtype != ZARYA_BF16) return "slot_attn_f32_kernel";
+  return plan_tc(desc, sm_count()).pair ? "slot_attn_pair_kernel" : "slot_attn_tc_kernel";
+}
+
 size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc) {
   if (check_desc(desc) != ZARYA_OK || check_attn_support(desc) != ZARYA_OK) return 0;
   if (desc->dtype != ZARYA_BF16) return 0;

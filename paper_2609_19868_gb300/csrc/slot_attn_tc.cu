@@ -1151,7 +1151,9 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   }
   // every barrier is initialised before any thread touches one
   __syncthreads();
-  if (warp == 3) {
+  // warp 1 holds the tensor memory, warp 3 issues the MMAs (its SM
+  // sub-partition's softmax warps measured least slowed by the issuer)
+  if (warp == 1) {
     tmem_alloc(&bars->tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -1222,7 +1224,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   if (!works) {
     if (code != 0 && pair == 0 && threadIdx.x == 0) record_error(p.err, code);
     grid_launch_dependents();
-    if (warp == 3) tmem_dealloc(tmem, kTmemCols);
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
     return;
   }
 
@@ -1239,7 +1241,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
                          smem_u32(smem + kPOffV), p, bars, b, kvh, 0, 0, nt, kv_end, lane, t_stage,
                          issued))
         drain_ring(bars->v_full, kPairStagesV, issued, lane);
-    } else if (warp == 1) {
+    } else if (warp == 3) {
       // ======================= MMA issuer (one elected lane) =======================
       bool ok = true;
       if (p.debug_stall) ok = wait_bar(&bars->stall, 0, bars, p);
@@ -1484,7 +1486,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   tc_fence_before();
   __syncthreads();
   if (*reinterpret_cast<volatile int*>(&bars->abort) != 0) {
-    if (warp == 1 && mma_issued) {
+    if (warp == 3 && mma_issued) {
       tc_commit_elect(&bars->drain);
       mbar_wait(&bars->drain, 0, kDrainNs, nullptr);
     }
@@ -1497,7 +1499,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
     tc_fence_before();
     __syncthreads();
   }
-  if (warp == 3) {
+  if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }

@@ -330,3 +330,18 @@ def test_top_p_rejects_invalid_calls(lib):
     # overlapping rows (stride below the vocabulary) are refused before anything runs
     short = _sdesc(vocab=1000, row_stride=992)
     assert lib.zarya_top_p(vp(FAKE), 0.9, ctypes.byref(short), None) == 1
+
+
+def test_kernel_name_follows_the_plan(lib):
+    """The paired kernel is planned for paged caches whose M-tile pairs fill
+    the GPU; contiguous caches, a forced key split or few pairs keep the
+    single-tile kernel; fp32 has its own; invalid descriptors name none."""
+    name = lambda d: lib.zarya_slot_attn_kernel(ctypes.byref(d)).decode()  # noqa: E731
+    paged = dict(batch=64, n_q_heads=32, n_kv_heads=8, page_size=16, cache_capacity=16640,
+                 n_pages=30000, max_rows=256, total_rows=8192)
+    assert name(_desc(**paged)) == "slot_attn_pair_kernel"
+    assert name(_desc(**dict(paged, kv_splits=2))) == "slot_attn_tc_kernel"
+    assert name(_desc(**dict(paged, batch=2))) == "slot_attn_tc_kernel"
+    assert name(_desc(**dict(paged, page_size=0, n_pages=0))) == "slot_attn_tc_kernel"
+    assert name(_desc(dtype=zb.FP32, head_dim=64)) == "slot_attn_f32_kernel"
+    assert name(_desc(batch=0)) == "none"
