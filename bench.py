@@ -421,6 +421,10 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
             kc, vc = base.k_cache.clone(), base.v_cache.clone()
             rots.append(session.upload(w, dev, caches=(kc, vc)))
     kernel = zb.slot_attn_kernel(base.desc)   # the kernel the plan launches
+    # kernels per step: the attention call's (a dispatch-order kernel first
+    # when the plan sorts its tiles; the fp32 path stages with an append), and
+    # the length commit
+    launches_per_step = zb.slot_attn_launches(base.desc) + (w.dtype != "bf16") + 1
     # The commit writes the advanced lengths into a second array (the
     # ping-pong a decoding loop would use), so every step starts from the same
     # prefix lengths: a stationary workload with no copy between steps.
@@ -614,6 +618,7 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
         "hbm_gbs": counts["attn_bytes"] / (attn_ms * 1e-3) / 1e9,
         "tflops": counts["flops"] / (attn_ms * 1e-3) / 1e12,
         "steps_per_s": replica_throughput(K, world, step_ms * K),
+        "launches_per_step": launches_per_step,
     }
     del rots, graphs, dev_in, base
     torch.cuda.synchronize()
@@ -771,9 +776,10 @@ def run_ours(args):
             "layers_28_steps_per_s": round(value / 28, 2),
             "layers_36_steps_per_s": round(value / 36, 2),
         },
-        # staged attention + length commit per step, in every timed region
-        "gpu_launches": 2 * K * s_n,
-        "gpu_launches_note": f"2 kernels per step x {K} steps x {s_n} timed regions",
+        # the attention call's kernels + the length commit, every timed region
+        "gpu_launches": head["launches_per_step"] * K * s_n,
+        "gpu_launches_note": f"{head['launches_per_step']} kernels per step x {K} steps x "
+                             f"{s_n} timed regions",
         "clocks": clocks,
     }
     if per_config:

@@ -131,9 +131,11 @@ typedef struct {
 /*
  * Bytes of scratch memory zarya_slot_attn needs for `desc` (0 if it needs
  * none). The workspace holds split-KV partial results and per-tile arrival
- * counters. It must be zero-filled once before its first use; every call
- * leaves the counters at zero again, so it can be reused by later calls on
- * the same stream. After a call that set the device error word, zero it again.
+ * counters (more than 3 key splits), or the dispatch order of the work tiles
+ * (slot_attn_pair_kernel taking several waves of CTAs). It must be zero-filled
+ * once before its first use; every call leaves the counters at zero again, so
+ * it can be reused by later calls on the same stream. After a call that set
+ * the device error word, zero it again.
  * Returns 0 as well when desc is invalid (zarya_slot_attn will reject it).
  */
 size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc);
@@ -148,6 +150,16 @@ size_t zarya_slot_attn_workspace_size(const zarya_attn_desc* desc);
  * device work.
  */
 const char* zarya_slot_attn_kernel(const zarya_attn_desc* desc);
+
+/*
+ * Kernels one zarya_slot_attn call launches for `desc` on the current device:
+ * 2 when the plan sorts its work tiles first (slot_attn_pair_kernel taking
+ * several waves of CTAs: a one-CTA kernel writes the longest-first dispatch
+ * order into the workspace, then the attention kernel follows it), else 1;
+ * 0 for a descriptor zarya_slot_attn would reject. zarya_slot_attn_staged
+ * with fp32 launches one more (the staging append). No device work.
+ */
+int32_t zarya_slot_attn_launches(const zarya_attn_desc* desc);
 
 /*
  * Slot attention (Sec. 5.2 steps 3 and 6): for every sequence b, query head

@@ -93,8 +93,14 @@ def load() -> ctypes.CDLL:
     dp = ctypes.POINTER(AttnDesc)
     lib.zarya_slot_attn_workspace_size.argtypes = [dp]
     lib.zarya_slot_attn_workspace_size.restype = sz
-    lib.zarya_slot_attn_kernel.argtypes = [dp]
-    lib.zarya_slot_attn_kernel.restype = ctypes.c_char_p
+    # plan queries (a library built before them lacks these two; every
+    # declared function's presence is checked by the tests)
+    if hasattr(lib, "zarya_slot_attn_kernel"):
+        lib.zarya_slot_attn_kernel.argtypes = [dp]
+        lib.zarya_slot_attn_kernel.restype = ctypes.c_char_p
+    if hasattr(lib, "zarya_slot_attn_launches"):
+        lib.zarya_slot_attn_launches.argtypes = [dp]
+        lib.zarya_slot_attn_launches.restype = i32
     lib.zarya_slot_attn.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, dp, vp]
     lib.zarya_slot_attn.restype = ctypes.c_int
     lib.zarya_slot_attn_staged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
@@ -199,6 +205,11 @@ def make_desc(*, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int, dty
 def slot_attn_kernel(desc: AttnDesc) -> str:
     """``zarya_slot_attn_kernel``: the kernel the plan for ``desc`` launches."""
     return load().zarya_slot_attn_kernel(ctypes.byref(desc)).decode()
+
+
+def slot_attn_launches(desc: AttnDesc) -> int:
+    """``zarya_slot_attn_launches``: kernels one attention call launches."""
+    return int(load().zarya_slot_attn_launches(ctypes.byref(desc)))
 
 
 def workspace_size(desc: AttnDesc) -> int:

@@ -38,6 +38,12 @@ struct TcParams {
   int m_tiles, splits;
   int cluster;        // 1: the splits of a tile form a cluster and merge through DSMEM
   int pair;           // 1: one CTA per pair of M-tiles (paged caches, no key split)
+  // Longest-first dispatch (no key split, several waves): the CTA at linear
+  // position pos serves KV head pos % Hkv of work item perm[pos / Hkv], item
+  // i being (sequence i / items, M-tile or pair i % items); nullptr: the grid's
+  // own order.
+  const int32_t* perm;
+  int items;          // work items per sequence (M-tiles, or pairs of them)
   float scale_log2;   // softmax scale * log2(e)
   uint64_t wait_ns;   // bound on every pipeline wait (global-timer nanoseconds)
   int debug_stall;    // 1: the MMA warp first waits on a barrier nothing completes
@@ -114,6 +120,11 @@ cudaError_t launch_verify_accept(const SampleCall& c, const int32_t* tokens, flo
 
 // Dynamic shared memory of the tensor-core kernel.
 size_t tc_smem_bytes();
+
+// Most work items one dispatch order can sort (B x items).
+constexpr int kMaxSchedItems = 4096;
+// Writes p.perm: the work items sorted by cost (M-tiles x key tiles), largest first.
+cudaError_t launch_schedule(const TcParams& p, cudaStream_t stream);
 
 cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map_k,
                                 const CUtensorMap& map_v, const TcParams& p,

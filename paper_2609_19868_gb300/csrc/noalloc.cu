@@ -70,15 +70,19 @@ zarya_status zarya_slot_attn_noalloc(const void* q, const void* k_cache, const v
   if (need > 0) {
     scratch = zarya::scratch_address(&ce);
     if (scratch == nullptr) return zarya::cuda_fail("looking up the scratch address", ce);
-    // The split counters sit at the end of the workspace layout and must
-    // start at zero; the array keeps whatever the last call left.
+    // The split counters, when the plan has them, sit at the end of the
+    // workspace layout and must start at zero; the array keeps whatever the
+    // last call left. (A dispatch order needs no clearing: it is rewritten
+    // by every call.)
     const size_t cnt_bytes = zarya::workspace_counter_bytes(desc);
-    if (cnt_bytes == 0 || cnt_bytes > need)
+    if (cnt_bytes > need)
       return zarya::cuda_fail("split counter layout does not fit the scratch plan",
                               cudaErrorInvalidValue);
-    ce = cudaMemsetAsync(static_cast<unsigned char*>(scratch) + (need - cnt_bytes), 0, cnt_bytes,
-                         stream);
-    if (ce != cudaSuccess) return zarya::cuda_fail("clearing the split counters", ce);
+    if (cnt_bytes > 0) {
+      ce = cudaMemsetAsync(static_cast<unsigned char*>(scratch) + (need - cnt_bytes), 0,
+                           cnt_bytes, stream);
+      if (ce != cudaSuccess) return zarya::cuda_fail("clearing the split counters", ce);
+    }
   }
   return zarya_slot_attn(q, k_cache, v_cache, cache_lens, page_table, n_slots, slot_len,
                          mask_mode, out, scratch, need > 0 ? zarya::kScratchBytes : 0, desc,

@@ -439,6 +439,18 @@ __device__ __forceinline__ void drain_ring(uint64_t* full, int stages, int issue
       mbar_wait(&full[i % stages], (i / stages) & 1, kDrainNs, nullptr);
 }
 
+// The work tile of the CTA at linear position pos under the schedule: item
+// perm[pos / Hkv] (sequence item / items, tile item % items), KV head
+// pos % Hkv. Returns false for an item outside [0, B x items).
+__device__ __forceinline__ bool scheduled_tile(const TcParams& p, int item, int pos, int& b,
+                                               int& kvh, int& t) {
+  if (item < 0 || item >= p.B * p.items) return false;
+  b = item / p.items;
+  t = item - b * p.items;
+  kvh = pos % p.Hkv;
+  return true;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                     const __grid_constant__ CUtensorMap map_k,
@@ -1117,10 +1129,12 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int pair = blockIdx.x;
-  const int bh = blockIdx.z;
-  const int b = bh / p.Hkv;
-  const int kvh = bh - b * p.Hkv;
+  // the work tile, from the grid or the schedule (read after the wait)
+  const int pos = blockIdx.z * gridDim.x + blockIdx.x;
+  int pair = blockIdx.x;
+  int b = blockIdx.z / p.Hkv;
+  int kvh = blockIdx.z - b * p.Hkv;
+  bool sched_ok = true;
 
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&map_q);
@@ -1160,6 +1174,8 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   if (warp == 0 || warp == 2) named_bar_arrive(kBarSetup, kThreads);
   // Inputs may be written by the kernel launched before this one.
   grid_dependency_wait();
+  if (p.perm != nullptr) sched_ok = scheduled_tile(p, p.perm[pos / p.Hkv], pos, b, kvh, pair);
+  if (!sched_ok) b = 0;   // reported below; no work is done
 
   // ---- per-sequence geometry (uniform over the CTA) ----
   const int P = p.cache_lens[b];
@@ -1169,8 +1185,10 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   const int row0 = p.q_row_offsets[b];
   const int row_end = p.q_row_offsets[b + 1];
   int code = 0;
-  if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL &&
-      mode != ZARYA_MASK_SLOT_INDEPENDENT)
+  if (!sched_ok)
+    code = ZARYA_DEVERR_ROWS;
+  else if (mode != ZARYA_MASK_BIDIR_BLOCK && mode != ZARYA_MASK_SLOT_CAUSAL &&
+           mode != ZARYA_MASK_SLOT_INDEPENDENT)
     code = ZARYA_DEVERR_MASK_MODE;
   else if (p.n_slots[b] < 1 || p.slot_len[b] < 1 || R > p.max_rows || row_end - row0 != R ||
            row0 < 0 || row_end > p.total_rows)
@@ -1222,7 +1240,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   const uint32_t tmem = (warp != 0 && warp != 2) ? bars->tmem_base : 0u;
   bool mma_issued = false;
   if (!works) {
-    if (code != 0 && pair == 0 && threadIdx.x == 0) record_error(p.err, code);
+    if (code != 0 && (pair == 0 || !sched_ok) && threadIdx.x == 0) record_error(p.err, code);
     grid_launch_dependents();
     if (warp == 1) tmem_dealloc(tmem, kTmemCols);
     return;
@@ -1505,9 +1523,80 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   }
 }
 
+// ---------------------------------------------------------------------------
+// Dispatch order. A launch of several waves runs its CTAs in grid order as SMs
+// free up, so a long work tile dispatched late sets the end of the launch
+// (serving_mix: SMs busy 85 % of the launch). For paired launches of several
+// waves this one-CTA kernel sorts the work items (sequence, M-tile or pair) by cost
+// (M-tiles x key tiles: the tile loop's work), largest first, ties in item
+// order, and the attention CTA at position pos serves item perm[pos / Hkv],
+// KV head pos % Hkv: the greedy longest-first order. Items a CTA would find
+// empty (or invalid: the attention kernel reports those) cost 0 and go last.
+constexpr int kSchedThreads = 1024;
+
+__global__ void __launch_bounds__(kSchedThreads) schedule_kernel(const TcParams p) {
+  __shared__ unsigned long long key[kMaxSchedItems];
+  grid_dependency_wait();
+  const int T = p.items;
+  const int N = p.B * T;
+  int n2 = 1;
+  while (n2 < N) n2 <<= 1;
+  const int rows_per_tile = kBlockM / p.g;
+  const int span = p.pair ? 2 : 1;   // M-tiles per item
+  for (int i = threadIdx.x; i < n2; i += kSchedThreads) {
+    unsigned long long k = ~0ull;
+    if (i < N) {
+      const int b = i / T, t = i - b * T;
+      const int P = p.cache_lens[b];
+      const long long R64 = static_cast<long long>(p.n_slots[b]) * p.slot_len[b];
+      const int mode = p.mask_mode[b];
+      uint32_t cost = 0;
+      if (P >= 0 && R64 >= 1 && R64 <= p.max_rows && P + R64 <= p.capacity) {
+        const int R = static_cast<int>(R64);
+        const int r0 = span * t * rows_per_tile;
+        if (r0 < R) {
+          const int m = min(span, (R - r0 + rows_per_tile - 1) / rows_per_tile);
+          const int r_hi = min(r0 + span * rows_per_tile, R) - 1;
+          const int kv_end = mode == ZARYA_MASK_BIDIR_BLOCK ? P + R : P + r_hi + 1;
+          cost = static_cast<uint32_t>(m) * static_cast<uint32_t>((kv_end + kBlockN - 1) / kBlockN) + 1;
+        }
+      }
+      k = (static_cast<unsigned long long>(0xFFFFFFFFu - cost) << 32) | static_cast<uint32_t>(i);
+    }
+    key[i] = k;
+  }
+  __syncthreads();
+  // bitonic sort, ascending key = descending cost
+  for (int size = 2; size <= n2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < n2; i += kSchedThreads) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool up = (i & size) == 0;
+          const unsigned long long a = key[i], c = key[j];
+          if ((a > c) == up) {
+            key[i] = c;
+            key[j] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  int32_t* perm = const_cast<int32_t*>(p.perm);
+  for (int k = threadIdx.x; k < N; k += kSchedThreads)
+    perm[k] = static_cast<int32_t>(key[k] & 0xFFFFFFFFull);
+  grid_launch_dependents();
+}
+
 }  // namespace
 
 size_t tc_smem_bytes() { return kSmemBytes; }
+
+cudaError_t launch_schedule(const TcParams& p, cudaStream_t stream) {
+  PdlLaunch l(dim3(1), dim3(kSchedThreads), 0, stream);
+  return cudaLaunchKernelEx(&l.cfg, schedule_kernel, p);
+}
 
 cudaError_t launch_slot_attn_tc(const CUtensorMap& map_q, const CUtensorMap& map_k,
                                 const CUtensorMap& map_v, const TcParams& p,

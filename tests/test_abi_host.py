@@ -345,3 +345,23 @@ def test_kernel_name_follows_the_plan(lib):
     assert name(_desc(**dict(paged, page_size=0, n_pages=0))) == "slot_attn_tc_kernel"
     assert name(_desc(dtype=zb.FP32, head_dim=64)) == "slot_attn_f32_kernel"
     assert name(_desc(batch=0)) == "none"
+
+
+def test_dispatch_order_is_planned_for_unsplit_multi_wave_launches(lib):
+    """A paired launch (paged cache) taking several waves of CTAs gets a
+    longest-first dispatch order: one more kernel and a workspace of one
+    int32 per work item; other plans get neither."""
+    wsz = lambda d: lib.zarya_slot_attn_workspace_size(ctypes.byref(d))  # noqa: E731
+    nl = lambda d: lib.zarya_slot_attn_launches(ctypes.byref(d))  # noqa: E731
+    paged = dict(batch=64, n_q_heads=32, n_kv_heads=8, page_size=16, cache_capacity=16640,
+                 n_pages=30000, max_rows=256, total_rows=8192)
+    d = _desc(**paged)                        # 64 x 4 pairs, x 8 heads: many waves
+    assert nl(d) == 2 and wsz(d) == (64 * 4 * 4 + 255) // 256 * 256
+    ragged = dict(batch=32, n_q_heads=32, n_kv_heads=8, cache_capacity=8320, max_rows=128,
+                  total_rows=4096)
+    assert nl(_desc(**ragged)) == 1 and wsz(_desc(**ragged)) == 0   # contiguous: grid order
+    assert nl(_desc(**dict(paged, kv_splits=1))) == 1      # forced split: single-tile kernel
+    assert nl(_desc(**dict(paged, batch=2))) == 1          # pairs do not fill the GPU
+    assert nl(_desc()) == 1 and wsz(_desc()) == 0        # 16 CTAs: one wave
+    assert nl(_desc(dtype=zb.FP32, head_dim=64)) == 1
+    assert nl(_desc(batch=0)) == 0
