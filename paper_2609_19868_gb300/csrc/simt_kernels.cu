@@ -74,8 +74,10 @@ __device__ __forceinline__ long long token_row(const int32_t* page_table, int pa
   return static_cast<long long>(page) * page_size + c % page_size;
 }
 
+constexpr int kF32Warps = 8;   // warps per CTA of the fp32 attention kernel
+
 template <int kPerLane>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(kF32Warps * 32)
 slot_attn_f32_kernel(const SimtParams p) {
   grid_dependency_wait();
   grid_launch_dependents();
@@ -104,34 +106,75 @@ slot_attn_f32_kernel(const SimtParams p) {
                    (static_cast<long long>(row0 + r) * p.Hq + h) * D;
   const float* kc = reinterpret_cast<const float*>(p.k_cache);
   const float* vc = reinterpret_cast<const float*>(p.v_cache);
-  float qv[kPerLane], o[kPerLane];
+  // This warp's query row in shared memory (every lane reads all of it).
+  __shared__ float4 qs[kF32Warps][D / 4];
+  float* qw = reinterpret_cast<float*>(qs[threadIdx.x >> 5]);
 #pragma unroll
-  for (int x = 0; x < kPerLane; ++x) {
-    qv[x] = q[lane + 32 * x];
-    o[x] = 0.f;
-  }
+  for (int x = 0; x < kPerLane; ++x) qw[lane + 32 * x] = q[lane + 32 * x];
+  __syncwarp();
+  // Online softmax over chunks of 32 visible keys (the earlier slots' hidden
+  // block rows [P, hide_hi) skipped): lane k scores key k of the chunk with a
+  // whole dot product, the warp takes the chunk's maximum and sum, and the
+  // chunk's weights are broadcast to accumulate O, lane l holding columns
+  // l, l + 32, ...
+  const int nv = P + (n_vis - hide_hi);
+  float o[kPerLane];
+#pragma unroll
+  for (int x = 0; x < kPerLane; ++x) o[x] = 0.f;
   float m = -INFINITY, l = 0.f;
-  for (int c = 0; c < n_vis; ++c) {
-    if (c == P && hide_hi > P) c = hide_hi;   // skip the hidden block rows
-    const long long tr =
-        token_row(p.page_table, p.page_size, p.max_pages, p.n_pages, p.capacity, b, c);
-    if (tr < 0) {
+  for (int base = 0; base < nv; base += 32) {
+    const int i = base + lane;
+    float s = -INFINITY;
+    long long row = 0;   // first element of this lane's key row (K and V)
+    bool bad = false;
+    if (i < nv) {
+      const int c = i < P ? i : i - P + hide_hi;
+      const long long tr =
+          token_row(p.page_table, p.page_size, p.max_pages, p.n_pages, p.capacity, b, c);
+      if (tr < 0) {
+        bad = true;
+      } else {
+        row = (tr * p.Hkv + j) * D;
+        const float4* k4 = reinterpret_cast<const float4*>(kc + row);
+        float dot0 = 0.f, dot1 = 0.f;
+#pragma unroll 8
+        for (int d = 0; d < D / 4; ++d) {
+          const float4 kv = k4[d];
+          const float4 qv = qs[threadIdx.x >> 5][d];
+          dot0 = fmaf(qv.x, kv.x, dot0);
+          dot1 = fmaf(qv.y, kv.y, dot1);
+          dot0 = fmaf(qv.z, kv.z, dot0);
+          dot1 = fmaf(qv.w, kv.w, dot1);
+        }
+        s = (dot0 + dot1) * p.scale;
+      }
+    }
+    if (__any_sync(0xffffffffu, bad)) {
       if (lane == 0) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
       return;
     }
-    const long long base = (tr * p.Hkv + j) * D;
-    float dot = 0.f;
+    float cm = s;
 #pragma unroll
-    for (int x = 0; x < kPerLane; ++x) dot = fmaf(qv[x], kc[base + lane + 32 * x], dot);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    const float s = dot * p.scale;
-    const float m_new = fmaxf(m, s);
+    for (int off = 16; off > 0; off >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
+    const float m_new = fmaxf(m, cm);
     const float corr = (m == -INFINITY) ? 0.f : expf(m - m_new);
-    const float w = expf(s - m_new);
-    l = l * corr + w;
+    const float w = (i < nv) ? expf(s - m_new) : 0.f;
+    float ws = w;
 #pragma unroll
-    for (int x = 0; x < kPerLane; ++x) o[x] = fmaf(w, vc[base + lane + 32 * x], o[x] * corr);
+    for (int off = 16; off > 0; off >>= 1) ws += __shfl_xor_sync(0xffffffffu, ws, off);
+    l = l * corr + ws;
+#pragma unroll
+    for (int x = 0; x < kPerLane; ++x) o[x] *= corr;
+    const int n = min(32, nv - base);
+#pragma unroll 16
+    for (int k = 0; k < 32; ++k) {
+      const float wk = __shfl_sync(0xffffffffu, w, k);
+      const long long rk = __shfl_sync(0xffffffffu, row, k);
+      if (k < n) {
+#pragma unroll
+        for (int x = 0; x < kPerLane; ++x) o[x] = fmaf(wk, vc[rk + lane + 32 * x], o[x]);
+      }
+    }
     m = m_new;
   }
   float* out = reinterpret_cast<float*>(p.out) + (static_cast<long long>(row0 + r) * p.Hq + h) * D;

@@ -265,3 +265,60 @@ def test_batching_leaves_each_sequence_bitwise_unchanged(zs):
         lo, hi = int(w.q_row_offsets[b]), int(w.q_row_offsets[b + 1])
         alone = _run(zs, _one_sequence(w, b), kv_splits=1).out
         assert torch.equal(full[lo:hi], alone), f"sequence {b}"
+
+
+def test_dispatch_order_is_longest_first_and_changes_no_byte(zs, oracle_mod):
+    """A paired launch of several waves first sorts its work items: the
+    workspace then holds a permutation of (sequence, pair) items in
+    non-increasing cost (M-tiles x key tiles, the tile loop's work; empty
+    items last), ties in item order, and the output matches the oracle. The
+    same batch in grid order (a forced split: the single-tile kernel, no
+    order) matches it too."""
+    session, zb = zs
+    w = wl.make("serving_mix", seed=11, B=40, prefix=("loguniform", 20, 900))
+    db = _run(zs, w)
+    assert zb.slot_attn_kernel(db.desc) == "slot_attn_pair_kernel"
+    assert zb.slot_attn_launches(db.desc) == 2
+    T = int(db.desc.max_rows * (w.Hq // w.Hkv) + 127) // 128
+    T = (T + 1) // 2
+    perm = db.workspace[: 4 * w.B * T].view(torch.int32).cpu().numpy()
+    assert sorted(perm.tolist()) == list(range(w.B * T))
+    rpt = 128 // (w.Hq // w.Hkv)
+    cost = []
+    for item in perm:
+        b, t = divmod(int(item), T)
+        R, P = int(w.R[b]), int(w.cache_lens[b])
+        r0 = 2 * t * rpt
+        if r0 >= R:
+            cost.append(0)
+            continue
+        m = min(2, -(-(R - r0) // rpt))
+        r_hi = min(r0 + 2 * rpt, R) - 1
+        kv = P + R if w.mask_mode[b] == 0 else P + r_hi + 1
+        cost.append(m * (-(-kv // 128)) + 1)
+    keys = [(-c, int(i)) for c, i in zip(cost, perm)]
+    assert keys == sorted(keys)
+    kc, vc = oracle_staged(oracle_mod, w)
+    ok, err, _ = tolerance_ok(db.out, oracle_full(oracle_mod, w, kc, vc), w.dtype)
+    assert ok, f"max|err|={err:.3e}"
+    grid_order = _run(zs, w, kv_splits=1)
+    assert zb.slot_attn_kernel(grid_order.desc) == "slot_attn_tc_kernel"
+    assert zb.slot_attn_launches(grid_order.desc) == 1
+    ok, err, _ = tolerance_ok(grid_order.out, oracle_full(oracle_mod, w, kc, vc), w.dtype)
+    assert ok, f"grid order: max|err|={err:.3e}"
+
+
+@pytest.mark.parametrize("D,page_size,mode", [(32, 0, 1), (64, 16, 0), (96, 16, 1), (128, 0, 2),
+                                              (128, 16, 2), (256, 0, 0)])
+def test_fp32_tier_shapes_and_masks_match_oracle(zs, oracle_mod, D, page_size, mode):
+    """The fp32 kernel over head sizes 32..256, contiguous and paged caches,
+    all three masks, prefixes from 0 (chunks of 32 keys with ragged tails)."""
+    w = wl.make("tiny_fp32", seed=13, B=5, Hq=8, Hkv=2, D=D, page_size=page_size,
+                prefix=("uniform", 0, 300), slot_len=("choice", [2, 3, 8]),
+                mode=("fixed", mode), accept=("upto_R",))
+    w = replace(w, cache_lens=w.cache_lens.copy())
+    w.cache_lens[0] = 0
+    db = _run(zs, w)
+    kc, vc = oracle_staged(oracle_mod, w)
+    ok, err, scale = tolerance_ok(db.out, oracle_full(oracle_mod, w, kc, vc), w.dtype)
+    assert ok, f"D={D} page={page_size} mode={mode}: max|err|={err:.3e} max|ref|={scale:.3f}"
