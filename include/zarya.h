@@ -504,15 +504,17 @@ zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
  * zarya_verify_accept, zarya_sample_rows with the same temperature) then runs
  * over the nucleus, each token with its usual noise, and reports
  * probabilities renormalised over it. The masses behind the boundary are
- * summed in 2^-40 fixed point, so the result does not depend on the order of
- * the GPU's additions; it can differ from exact arithmetic only where the
- * mass at a boundary lies within about 1e-6 of top_p.
+ * summed in fixed point (each token's mass to 2^-21 of itself), so the result
+ * does not depend on the order of the GPU's additions; it can differ from
+ * exact arithmetic only where the mass at a boundary lies within about 1e-6 of
+ * top_p.
  *  logits   [desc->total_rows, desc->row_stride] of desc->dtype (read and
  *           written; 16-byte aligned); rows of no sequence are untouched
  *  top_p    in (0, 1); top_p >= 1 returns at once (nothing to cut)
  * desc supplies batch, vocab, dtype, total_rows, row_stride, row_offsets and
  * temperature; its other fields are checked as for zarya_draft_select.
- * Returns ZARYA_ERR_INVALID_ARG for top_p <= 0 or NaN.
+ * Returns ZARYA_ERR_INVALID_ARG for top_p <= 0 or NaN, and
+ * ZARYA_ERR_UNSUPPORTED for a vocabulary above 520,192 tokens.
  */
 zarya_status zarya_top_p(void* logits, float top_p, const zarya_sample_desc* desc,
                          zarya_stream_t stream);

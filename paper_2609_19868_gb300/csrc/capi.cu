@@ -633,6 +633,7 @@ zarya_status zarya_top_p(void* logits, float top_p, const zarya_sample_desc* des
   if (st != ZARYA_OK) return st;
   if (!logits || !aligned16(logits)) return ZARYA_ERR_INVALID_ARG;
   if (!(top_p > 0.f)) return ZARYA_ERR_INVALID_ARG;   // also NaN
+  if (desc->vocab > kNucleusMaxVocab) return ZARYA_ERR_UNSUPPORTED;
   if (top_p >= 1.f) return ZARYA_OK;                  // the nucleus is the whole vocabulary
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   cudaError_t ce = select_device(stream, logits);

@@ -5,21 +5,36 @@
 // it, hold at least top_p of the row's probability softmax(x / T). The draws
 // that follow then run over the nucleus with renormalised probabilities.
 //
-// One CTA per row. x* is found by radix descent over the order-preserving
-// integer key of the logit (sign-flipped bits; 16 bits for bf16, 32 for
-// fp32), 8 bits per pass: a pass adds each qualifying element's mass
-// exp((x - m) / T) to a 256-bin histogram of its next key digit, and the bin
-// where the mass counted from the top reaches top_p of the total fixes that
-// digit. Masses are summed in 2^-40 fixed point (64-bit integers), so the sums,
-// and with them the boundary, do not depend on the order of the atomics.
-// The masses differ from exact ones by the fp32 exponent argument's rounding
-// (below 1e-6 relative for any token within 2^20 of the maximum's mass), the
-// approximate exp2 (2^-22) and the truncation to 2^-40 (masses below that count
-// as zero): a kept set can differ from the exact one only where the mass at
-// its boundary lies within about 1e-6 of top_p. Each lane adds into its own slot
-// of each bin (no two lanes of a warp share a word). The row is read, in
-// 16-byte vectors, once for its maximum, once per digit and once for the
-// masking writes.
+// One CTA per row, no atomics. With a = (x - m) log2(e) / T (one fused
+// multiply-add, monotone in x; m the row's maximum) a token's mass relative
+// to the maximum's is 2^a. Stage 1 sorts the tokens into one-octave mass
+// bins, j = floor(-a) for a in (-42, 0] (lighter tokens count as massless);
+// since j falls as x grows, each bin holds a contiguous range of logit
+// values. Every thread adds its tokens' masses into private slots, the slots
+// are summed in a fixed order, and the bin where the mass counted from the
+// top reaches top_p of the total contains x*. One warp then finds that bin's
+// range of order-preserving logit keys (sign-flipped bits; 16 bits for bf16,
+// 32 for fp32) by a 32-way search over the monotone bin function, a pass over
+// the row gathers the keys in that range into shared memory (each warp its
+// own segment, placed by ballots), and stage 2 runs a radix descent over them,
+// 4 bits of the key offset per level, again with private slots per thread: a
+// level sums each candidate's mass into its digit, and the digit where the
+// mass counted from the top reaches top_p is fixed. A row whose bin holds more
+// keys than the shared memory takes the descent's levels over the row instead.
+//
+// Masses are fixed point relative to their bin: a token of bin j adds
+// floor(2^(a + j + 22)) (between 2^21 and 2^22) in units of 2^-(j + 22), and
+// the integer sums are scaled to doubles only for the comparisons, so the
+// boundary does not depend on the order of the GPU's additions (a thread's
+// slots hold at most 1023 tokens, so 32 bits never overflow). The masses
+// differ from exact ones by the fp32 exponent argument's rounding (below 1e-6
+// relative for any token within 2^20 of the maximum's mass), the approximate
+// exp2 (2^-22) and the truncation (below 2^-21 relative; tokens under 2^-42 of
+// the maximum count as zero): a kept set can differ from the exact one only
+// where the mass at its boundary lies within about 1e-6 of top_p. The row is
+// read, in 16-byte vectors with several in flight per thread, once for its
+// maximum, once for the mass bins, once to gather the candidates and once for
+// the masking writes; after the first read it sits in L2.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -34,12 +49,33 @@ namespace {
 
 constexpr int kNucThreads = 512;
 constexpr int kNucWarps = kNucThreads / 32;
-// One histogram per CTA with a private slot per lane: bin b, lane l at
-// hist[b * kHistStride + l]. No two lanes of a warp ever add to the same
-// word (a warp's adds never serialise on an address, whatever the digits),
-// and the padding slot makes the per-bin sums below bank-conflict free.
-constexpr int kHistStride = 33;
-constexpr size_t kNucSmem = 256 * kHistStride * sizeof(unsigned long long);
+constexpr int kNucUnroll = 4;   // 16-byte loads in flight per thread
+// Mass bins: bin j holds the tokens with a in (-j - 1, -j].
+constexpr int kMassBins = 42;
+constexpr float kMassFloor = -42.f;
+constexpr float kMassFloorUp = -41.999996185302734375f;   // the float just above -42
+// floor(-c) for c in [-42, 0] from the bits of fma_rz(c, -1, 1.5 * 2^23)
+constexpr float kBinMagic = 12582912.f;
+constexpr uint32_t kBinMagicBits = 0x4B400000u;
+// The descent's digits: 4 bits of the key offset per level.
+constexpr int kDigitBits = 4;
+constexpr int kDigits = 1 << kDigitBits;
+// Shared memory: stage 1's private slots (bin j, thread t at j * kNucThreads
+// + t, 32 bits); afterwards the descent's private slots (digit k, thread t at
+// k * kNucThreads + t) and, behind them, the candidates' keys, one segment of
+// kCandBytes / kNucWarps bytes per warp.
+constexpr size_t kNucSmem = static_cast<size_t>(kMassBins) * kNucThreads * sizeof(uint32_t);
+constexpr size_t kDigitBytes = static_cast<size_t>(kDigits) * kNucThreads * sizeof(uint32_t);
+constexpr size_t kCandBytes = kNucSmem - kDigitBytes;
+// A thread adds at most this many tokens into a 32-bit slot (each at most
+// 2^22 + 1): up to ceil(V / (kPerVec * kNucThreads)) vectors of kPerVec and
+// one tail token, which kNucleusMaxVocab keeps within it.
+constexpr int kMaxTokensPerThread = 1023;
+static_assert(((kNucleusMaxVocab / 8 + kNucThreads - 1) / kNucThreads) * 8 + 1 <= kMaxTokensPerThread &&
+                  ((kNucleusMaxVocab / 4 + kNucThreads - 1) / kNucThreads) * 4 + 1 <= kMaxTokensPerThread,
+              "a thread's 32-bit mass slots could overflow");
+static_assert(static_cast<unsigned long long>(kMaxTokensPerThread) * ((1u << 22) + 1u) < (1ull << 32),
+              "a thread's 32-bit mass slots could overflow");
 
 __device__ __forceinline__ float nuc_ex2(float x) {
   float y;
@@ -47,52 +83,118 @@ __device__ __forceinline__ float nuc_ex2(float x) {
   return y;
 }
 
-// floor(e * 2^40) for e in [0, 1] (the mass in 2^-40 fixed point), from the
-// float's fields: e = mant * 2^(ex - 23) with the implicit bit in mant.
-// NaN (never a mass of a finite logit) counts as 0.
-__device__ __forceinline__ unsigned long long mass_fixed(float e) {
-  const uint32_t u = __float_as_uint(e);
-  const int sh = static_cast<int>(u >> 23) - 127 + 40 - 23;
-  if (sh > 17 || sh <= -24) return 0ull;   // NaN / above 1, or below 2^-40
-  const unsigned long long mant = (u & 0x7FFFFFu) | 0x800000u;
-  return sh >= 0 ? (mant << sh) : (mant >> (-sh));
+// 2^-(j + 22) as a double (bin j's unit).
+__device__ __forceinline__ double bin_unit(int j) {
+  return __longlong_as_double(static_cast<long long>(1023 - j - 22) << 52);
 }
 
-// Order-preserving key of a logit and the logit of a key.
-__device__ __forceinline__ uint32_t logit_key(uint16_t b) {
-  return b ^ ((b & 0x8000u) ? 0xFFFFu : 0x8000u);
-}
-__device__ __forceinline__ uint32_t logit_key(uint32_t b) {
-  return b ^ ((b & 0x80000000u) ? 0xFFFFFFFFu : 0x80000000u);
-}
-
-template <typename TBits>
-__device__ __forceinline__ float bits_to_float(TBits b) {
-  if (sizeof(TBits) == 2) return __uint_as_float(static_cast<uint32_t>(b) << 16);
-  return __uint_as_float(static_cast<uint32_t>(b));
-}
-
-// The logits of 16-byte vector w.
-template <typename TBits>
-struct Vec16 {
-  static constexpr int kN = 16 / sizeof(TBits);
-  TBits e[kN];
-  __device__ __forceinline__ explicit Vec16(const uint4& w) {
-    const TBits* p = reinterpret_cast<const TBits*>(&w);
-#pragma unroll
-    for (int k = 0; k < kN; ++k) e[k] = p[k];
-  }
+// A token's mass in its bin's units, and its bin. The same arithmetic decides
+// the bins in stage 1, in the key-range search and in stage 2.
+struct Mass {
+  uint32_t q;   // 0 for a massless token (a <= -42, or NaN)
+  uint32_t j;
 };
+__device__ __forceinline__ Mass token_mass(float x, float k2, float neg_mk) {
+  const float a = fmaf(x, k2, neg_mk);
+  const float c = fminf(fmaxf(a, kMassFloorUp), 0.f);
+  const uint32_t j = __float_as_uint(__fmaf_rz(c, -1.f, kBinMagic)) - kBinMagicBits;
+  // e = 2^c lies in [2^-(j+1), 2^-j] up to the approximation: its 24-bit
+  // significand shifted to the units of 2^-(j + 22)
+  const uint32_t u = __float_as_uint(nuc_ex2(c));
+  const uint32_t r = min(128u - (u >> 23) - j, 31u);
+  const uint32_t q = ((u & 0x7FFFFFu) | 0x800000u) >> r;
+  return Mass{a > kMassFloor ? q : 0u, j};
+}
+
+// The bin of a logit (kMassBins for a massless one): token_mass's bin test.
+__device__ __forceinline__ int token_bin(float x, float k2, float neg_mk) {
+  const float a = fmaf(x, k2, neg_mk);
+  if (!(a > kMassFloor)) return kMassBins;
+  const float c = fminf(fmaxf(a, kMassFloorUp), 0.f);
+  return static_cast<int>(__float_as_uint(__fmaf_rz(c, -1.f, kBinMagic)) - kBinMagicBits);
+}
+
+// Order-preserving key of a logit given as fp32 bits (bf16 logits widened),
+// kKeyBits wide, and the fp32 bits of a key.
+template <int kKeyBits>
+__device__ __forceinline__ uint32_t logit_key(uint32_t f) {
+  const uint32_t k = f ^ (static_cast<uint32_t>(static_cast<int32_t>(f) >> 31) | 0x80000000u);
+  return k >> (32 - kKeyBits);
+}
+template <int kKeyBits>
+__device__ __forceinline__ uint32_t key_bits(uint32_t key) {
+  const uint32_t k = key << (32 - kKeyBits);
+  return (k & 0x80000000u) ? (k ^ 0x80000000u) : ~k & (0xFFFFFFFFu << (32 - kKeyBits));
+}
+
+// Calls f(fp32 bits) for each logit of a 16-byte vector.
+template <typename TBits, typename F>
+__device__ __forceinline__ void each_logit(const uint4& v, F&& f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    if (sizeof(TBits) == 2) {
+      f(w[k] << 16);
+      f(w[k] & 0xFFFF0000u);
+    } else {
+      f(w[k]);
+    }
+  }
+}
 
 template <typename TBits>
-__global__ void __launch_bounds__(kNucThreads) nucleus_kernel(const NucleusParams a) {
+__device__ __forceinline__ uint32_t widen(TBits b) {
+  return sizeof(TBits) == 2 ? static_cast<uint32_t>(b) << 16 : static_cast<uint32_t>(b);
+}
+
+// Calls f(w, i) on this thread's 16-byte vectors i = tid, tid + kNucThreads,
+// ... of v[0, n), with kNucUnroll loads in flight before the first is used.
+template <typename F>
+__device__ __forceinline__ void for_each_vec(const uint4* v, int n, int tid, F&& f) {
+  int i = tid;
+  for (; i + (kNucUnroll - 1) * kNucThreads < n; i += kNucUnroll * kNucThreads) {
+    uint4 w[kNucUnroll];
+#pragma unroll
+    for (int u = 0; u < kNucUnroll; ++u) w[u] = v[i + u * kNucThreads];
+#pragma unroll
+    for (int u = 0; u < kNucUnroll; ++u) f(w[u], i + u * kNucThreads);
+  }
+  for (; i < n; i += kNucThreads) f(v[i], i);
+}
+
+// The smallest key in [lo, hi] whose pred holds, hi + 1 if none; pred is
+// monotone (false ... false true ... true). Called by one whole warp; every
+// lane returns the same key.
+template <typename P>
+__device__ __forceinline__ uint32_t first_true_key(uint32_t lo, uint32_t hi, int lane, P&& pred) {
+  uint64_t a = lo, b = static_cast<uint64_t>(hi) + 1;   // the answer lies in [a, b]
+  while (a < b) {
+    const uint64_t step = (b - a + 31) >> 5;
+    const uint64_t probe = a + static_cast<uint64_t>(lane) * step;
+    const bool p = probe < b && pred(static_cast<uint32_t>(probe));
+    const unsigned bal = __ballot_sync(0xffffffffu, p);
+    const int last = 31 - __clz(__ballot_sync(0xffffffffu, probe < b));   // the last lane with a probe
+    const int f = bal ? __ffs(bal) - 1 : last + 1;   // the first lane whose probe holds
+    if (f == 0) return static_cast<uint32_t>(a);
+    const uint64_t na = a + static_cast<uint64_t>(f - 1) * step + 1;
+    b = f <= last ? a + static_cast<uint64_t>(f) * step : b;
+    a = na;
+  }
+  return static_cast<uint32_t>(a);
+}
+
+template <typename TBits>
+__global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusParams a) {
   constexpr int kKeyBits = 8 * static_cast<int>(sizeof(TBits));
   constexpr int kPerVec = 16 / static_cast<int>(sizeof(TBits));
-  extern __shared__ unsigned long long hist[];   // [256][kHistStride]
-  __shared__ unsigned long long bins[256];
+  constexpr int kSegKeys = static_cast<int>(kCandBytes / sizeof(TBits)) / kNucWarps;
+  extern __shared__ __align__(16) uint32_t smem[];
+  __shared__ unsigned long long bins[kMassBins];
   __shared__ float s_max[kNucWarps];
-  __shared__ uint32_t s_prefix;
-  __shared__ unsigned long long s_above, s_total;
+  __shared__ int s_seg[kNucWarps];
+  __shared__ int s_pick, s_over;
+  __shared__ uint32_t s_klo, s_khi, s_prefix;
+  __shared__ double s_above, s_target;
   grid_dependency_wait();
   grid_launch_dependents();
   const int g = blockIdx.x;
@@ -105,14 +207,22 @@ __global__ void __launch_bounds__(kNucThreads) nucleus_kernel(const NucleusParam
   const int nvec = V / kPerVec;
   const int tail0 = nvec * kPerVec;
 
-  // the row's maximum
+  // the row's maximum (NaN ignored)
   float m = -INFINITY;
-  for (int i = tid; i < nvec; i += kNucThreads) {
-    const Vec16<TBits> w(row4[i]);
-#pragma unroll
-    for (int k = 0; k < kPerVec; ++k) m = fmaxf(m, bits_to_float(w.e[k]));
+  if constexpr (sizeof(TBits) == 2) {
+    __nv_bfloat162 m2 = __float2bfloat162_rn(-INFINITY);
+    for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
+      const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+      m2 = __hmax2(m2, __hmax2(__hmax2(h[0], h[1]), __hmax2(h[2], h[3])));
+    });
+    m = fmaxf(__low2float(m2), __high2float(m2));
+  } else {
+    for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
+      m = fmaxf(m, fmaxf(fmaxf(__uint_as_float(v.x), __uint_as_float(v.y)),
+                         fmaxf(__uint_as_float(v.z), __uint_as_float(v.w))));
+    });
   }
-  for (int v = tail0 + tid; v < V; v += kNucThreads) m = fmaxf(m, bits_to_float(row[v]));
+  for (int v = tail0 + tid; v < V; v += kNucThreads) m = fmaxf(m, __uint_as_float(widen(row[v])));
 #pragma unroll
   for (int d = 16; d >= 1; d >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, d));
   if (lane == 0) s_max[warp] = m;
@@ -120,90 +230,213 @@ __global__ void __launch_bounds__(kNucThreads) nucleus_kernel(const NucleusParam
   m = s_max[0];
   for (int w = 1; w < kNucWarps; ++w) m = fmaxf(m, s_max[w]);
   if (!(m > -INFINITY)) return;   // every logit -inf (or NaN): nothing to cut
+  const float k2 = a.k2, neg_mk = -m * a.k2;
 
-  const float neg_mk = -m * a.k2;
-  uint32_t prefix = 0;
-  unsigned long long above = 0;   // mass of the keys above the current prefix's range
-  for (int level = 0; level < kKeyBits / 8; ++level) {
-    const int shift = kKeyBits - 8 * (level + 1);
-    for (int i = tid; i < 256 * kHistStride; i += kNucThreads) hist[i] = 0ull;
-    __syncthreads();
-    auto add = [&](TBits b) {
-      const uint32_t key = logit_key(b);
-      if (level > 0 && (key >> (shift + 8)) != prefix) return;
-      const unsigned long long q = mass_fixed(nuc_ex2(fmaf(bits_to_float(b), a.k2, neg_mk)));
-      if (q != 0ull) atomicAdd(&hist[((key >> shift) & 255u) * kHistStride + lane], q);
-    };
-    for (int i = tid; i < nvec; i += kNucThreads) {
-      const Vec16<TBits> w(row4[i]);
+  // Stage 1: the mass bins in private slots.
+  uint32_t* own = smem + tid;
 #pragma unroll
-      for (int k = 0; k < kPerVec; ++k) add(w.e[k]);
-    }
-    for (int v = tail0 + tid; v < V; v += kNucThreads) add(row[v]);
-    __syncthreads();
-    if (tid < 256) {
-      unsigned long long t = 0;
-#pragma unroll 8
-      for (int l = 0; l < 32; ++l) t += hist[tid * kHistStride + l];
-      bins[tid] = t;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      if (level == 0) {
-        unsigned long long tot = 0;
-        for (int b = 0; b < 256; ++b) tot += bins[b];
-        s_total = tot;
-      }
-      const double target = static_cast<double>(a.top_p) * static_cast<double>(s_total);
-      unsigned long long cum = above;
-      int pick = -1, lowest = -1;
-      for (int b = 255; b >= 0; --b) {
-        const unsigned long long h = bins[b];
-        if (h == 0ull) continue;
-        lowest = b;
-        if (static_cast<double>(cum + h) >= target) {
-          pick = b;
+  for (int j = 0; j < kMassBins; ++j) own[j * kNucThreads] = 0u;
+  auto add_mass = [&](uint32_t f) {
+    const Mass s = token_mass(__uint_as_float(f), k2, neg_mk);
+    own[s.j * kNucThreads] += s.q;
+  };
+  for_each_vec(row4, nvec, tid, [&](const uint4& v, int) { each_logit<TBits>(v, add_mass); });
+  for (int v = tail0 + tid; v < V; v += kNucThreads) add_mass(widen(row[v]));
+  __syncthreads();
+  for (int j = warp; j < kMassBins; j += kNucWarps) {   // fixed summation order
+    unsigned long long t = 0;
+    for (int i = lane; i < kNucThreads; i += 32) t += smem[j * kNucThreads + i];
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
+    if (lane == 0) bins[j] = t;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    double tot = 0.0;
+#pragma unroll 1
+    for (int j = 0; j < kMassBins; ++j) tot += static_cast<double>(bins[j]) * bin_unit(j);
+    const double target = static_cast<double>(a.top_p) * tot;
+    int pick = -1, lowest = -1;
+    double cum = 0.0;
+    if (tot > 0.0) {
+#pragma unroll 1
+      for (int j = 0; j < kMassBins; ++j) {
+        if (bins[j] == 0ull) continue;
+        const double h = static_cast<double>(bins[j]) * bin_unit(j);
+        lowest = j;
+        if (cum + h >= target) {
+          pick = j;
           break;
         }
         cum += h;
       }
       if (pick < 0) {   // the target is beyond the mass (rounding): keep down to the lowest bin
-        pick = lowest < 0 ? 0 : lowest;
-        cum = above;
-        for (int b = 255; b > pick; --b) cum += bins[b];
+        pick = lowest;
+        cum = 0.0;
+#pragma unroll 1
+        for (int j = 0; j < pick; ++j) cum += static_cast<double>(bins[j]) * bin_unit(j);
       }
-      s_prefix = (prefix << 8) | static_cast<uint32_t>(pick);
-      s_above = cum;
+    }
+    s_pick = pick;
+    s_above = cum;
+    s_target = target;
+    s_over = 0;
+  }
+  __syncthreads();
+  const int jbin = s_pick;
+  if (jbin < 0) return;   // no token has mass (a +inf logit): nothing to cut
+
+  // The key range of bin jbin (the bin falls as the key grows; NaN keys lie
+  // outside [key(-inf), key(+inf)]).
+  if (warp == 0) {
+    const uint32_t lo = logit_key<kKeyBits>(0xFF800000u), hi = logit_key<kKeyBits>(0x7F800000u);
+    auto bin_of = [&](uint32_t key) {
+      return token_bin(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk);
+    };
+    const uint32_t klo = first_true_key(lo, hi, lane, [&](uint32_t k) { return bin_of(k) <= jbin; });
+    const uint32_t kend = first_true_key(lo, hi, lane, [&](uint32_t k) { return bin_of(k) < jbin; });
+    if (lane == 0) {
+      s_klo = klo;
+      s_khi = kend - 1;
+    }
+  }
+  __syncthreads();
+  const uint32_t klo = s_klo, range = s_khi - s_klo;
+  uint32_t prefix = 0;   // the key offset of x* above the current level
+  if (range > 0) {
+    // Gather the keys of the bin into this warp's segment. The loop runs the
+    // same number of times in every lane of the warp (ballots need all 32).
+    TBits* seg = reinterpret_cast<TBits*>(reinterpret_cast<unsigned char*>(smem) + kDigitBytes) +
+                 warp * kSegKeys;
+    int cnt = 0;
+    auto gather = [&](uint32_t f, bool valid) {
+      const uint32_t key = logit_key<kKeyBits>(f);
+      const bool in = valid && key - klo <= range;
+      const unsigned bal = __ballot_sync(0xffffffffu, in);
+      const int pos = cnt + __popc(bal & ((1u << lane) - 1u));
+      if (in && pos < kSegKeys) seg[pos] = static_cast<TBits>(key);
+      cnt += __popc(bal);
+    };
+    const int warp0 = tid - lane;
+    for (int i0 = warp0; i0 < nvec; i0 += kNucUnroll * kNucThreads) {
+      uint4 w[kNucUnroll];
+#pragma unroll
+      for (int u = 0; u < kNucUnroll; ++u) {
+        const int i = i0 + u * kNucThreads + lane;
+        w[u] = i < nvec ? row4[i] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kNucUnroll; ++u) {
+        const bool valid = i0 + u * kNucThreads + lane < nvec;
+        each_logit<TBits>(w[u], [&](uint32_t f) { gather(f, valid); });
+      }
+    }
+    if (warp == 0) {   // the scalar tail (fewer than kPerVec logits)
+      const bool valid = tail0 + lane < V;
+      gather(valid ? widen(row[tail0 + lane]) : 0u, valid);
+    }
+    if (lane == 0) {
+      s_seg[warp] = min(cnt, kSegKeys);
+      if (cnt > kSegKeys) s_over = 1;
     }
     __syncthreads();
-    prefix = s_prefix;
-    above = s_above;
-    __syncthreads();   // hist is cleared by the next level
+    const bool over = s_over != 0;
+    const int n_mine = s_seg[warp];
+
+    // Stage 2: the radix descent over d = key - klo, kDigitBits per level,
+    // over the gathered keys (or the row, when a segment overflowed).
+    const int nbits = 32 - __clz(range);
+    const int levels = (nbits + kDigitBits - 1) / kDigitBits;
+    const double unit = bin_unit(jbin), target = s_target;
+    double above = s_above;   // mass of the tokens above the current range
+    for (int level = 0; level < levels; ++level) {
+      const int shift = kDigitBits * (levels - 1 - level);
+#pragma unroll
+      for (int k = 0; k < kDigits; ++k) own[k * kNucThreads] = 0u;
+      auto add = [&](uint32_t key) {
+        const uint32_t d = key - klo;
+        if (d > range) return;
+        if (level > 0 && (d >> (shift + kDigitBits)) != prefix) return;
+        const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk);
+        own[((d >> shift) & (kDigits - 1)) * kNucThreads] += s.q;
+      };
+      if (!over) {
+        for (int e = lane; e < n_mine; e += 32) add(seg[e]);
+      } else {
+        for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
+          each_logit<TBits>(v, [&](uint32_t f) { add(logit_key<kKeyBits>(f)); });
+        });
+        for (int v = tail0 + tid; v < V; v += kNucThreads) add(logit_key<kKeyBits>(widen(row[v])));
+      }
+      __syncthreads();
+      if (warp < kDigits) {   // digit `warp`'s total, in a fixed order
+        unsigned long long t = 0;
+        for (int i = lane; i < kNucThreads; i += 32) t += smem[warp * kNucThreads + i];
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
+        if (lane == 0) bins[warp] = t;
+      }
+      __syncthreads();
+      if (tid == 0) {
+        double cum = above;
+        int pick = -1, lowest = -1;
+#pragma unroll 1
+        for (int k = kDigits - 1; k >= 0; --k) {
+          if (bins[k] == 0ull) continue;
+          const double h = static_cast<double>(bins[k]) * unit;
+          lowest = k;
+          if (cum + h >= target) {
+            pick = k;
+            break;
+          }
+          cum += h;
+        }
+        if (pick < 0) {   // the target is beyond the mass (rounding): keep down to the lowest digit
+          pick = lowest < 0 ? 0 : lowest;
+          cum = above;
+#pragma unroll 1
+          for (int k = kDigits - 1; k > pick; --k) cum += static_cast<double>(bins[k]) * unit;
+        }
+        s_prefix = (prefix << kDigitBits) | static_cast<uint32_t>(pick);
+        s_above = cum;
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      above = s_above;
+    }
   }
-  // prefix is now the key of x*: every logit below it becomes -inf
-  const TBits neg_inf = sizeof(TBits) == 2 ? static_cast<TBits>(0xFF80u)
-                                           : static_cast<TBits>(0xFF800000u);
+
+  // x*'s key is klo + prefix: every logit below it becomes -inf
+  const uint32_t xkey = klo + prefix;
   uint4* wrow4 = reinterpret_cast<uint4*>(row);
-  for (int i = tid; i < nvec; i += kNucThreads) {
-    uint4 w = wrow4[i];
-    TBits* e = reinterpret_cast<TBits*>(&w);
+  for_each_vec(row4, nvec, tid, [&](const uint4& v, int i) {
+    uint32_t w[4] = {v.x, v.y, v.z, v.w};
     bool cut = false;
 #pragma unroll
-    for (int k = 0; k < kPerVec; ++k)
-      if (logit_key(e[k]) < prefix) {
-        e[k] = neg_inf;
-        cut = true;
+    for (int k = 0; k < 4; ++k) {
+      if constexpr (sizeof(TBits) == 2) {
+        const bool cl = logit_key<16>(w[k] << 16) < xkey;
+        const bool ch = logit_key<16>(w[k] & 0xFFFF0000u) < xkey;
+        w[k] = (cl ? 0xFF80u : (w[k] & 0xFFFFu)) | (ch ? 0xFF800000u : (w[k] & 0xFFFF0000u));
+        cut = cut || cl || ch;
+      } else {
+        const bool c = logit_key<32>(w[k]) < xkey;
+        w[k] = c ? 0xFF800000u : w[k];
+        cut = cut || c;
       }
-    if (cut) wrow4[i] = w;
-  }
+    }
+    if (cut) wrow4[i] = make_uint4(w[0], w[1], w[2], w[3]);
+  });
+  const TBits neg_inf = sizeof(TBits) == 2 ? static_cast<TBits>(0xFF80u)
+                                           : static_cast<TBits>(0xFF800000u);
   for (int v = tail0 + tid; v < V; v += kNucThreads)
-    if (logit_key(row[v]) < prefix) row[v] = neg_inf;
+    if (logit_key<kKeyBits>(widen(row[v])) < xkey) row[v] = neg_inf;
 }
 
 }  // namespace
 
 cudaError_t launch_nucleus(const NucleusParams& p, cudaStream_t stream) {
-  // the histogram's dynamic shared memory is above the default 48 KB limit
+  // the private slots' dynamic shared memory is above the default 48 KB limit
   constexpr int kMaxDevices = 64;
   static int configured[kMaxDevices] = {};
   int dev = 0;

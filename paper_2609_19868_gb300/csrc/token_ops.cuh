@@ -45,6 +45,9 @@ struct NucleusParams {
   int bf16;
 };
 
+// The largest vocabulary the top_p kernel takes (its per-thread 32-bit mass
+// sums stay below 2^32 up to it).
+constexpr int kNucleusMaxVocab = 520192;
 cudaError_t launch_nucleus(const NucleusParams& p, cudaStream_t stream);
 
 // Reordering / restoration of [B, max_len] token rows.

@@ -330,6 +330,9 @@ def test_top_p_rejects_invalid_calls(lib):
     # overlapping rows (stride below the vocabulary) are refused before anything runs
     short = _sdesc(vocab=1000, row_stride=992)
     assert lib.zarya_top_p(vp(FAKE), 0.9, ctypes.byref(short), None) == 1
+    # the kernel's 32-bit mass sums hold up to 520,192 tokens a row
+    big = _sdesc(vocab=520_200, row_stride=520_200)
+    assert lib.zarya_top_p(vp(FAKE), 0.9, ctypes.byref(big), None) == 2
 
 
 def test_kernel_name_follows_the_plan(lib):

@@ -131,3 +131,59 @@ def test_draws_after_top_p_stay_in_the_nucleus(zb, T):
             assert abs(z[tok[g]] - z[want]) < 1e-4 * (1 + abs(z[want]))
         p_ref = nuc.row_probability(xg, int(tok[g]), T, 0.6)
         assert abs(prob[g] - p_ref) < 1e-5 + 1e-4 * p_ref
+
+
+def _shaped_rows(rng, V):
+    """Rows whose masses sit in one mass bin, in every bin, or at its edges."""
+    flat = np.full(V, 1.25, dtype=np.float32)                        # every token equal
+    plateau = np.full(V, -3.0, dtype=np.float32)                      # a plateau and a few peaks
+    plateau[rng.choice(V, 7, replace=False)] = rng.uniform(2.0, 6.0, 7).astype(np.float32)
+    wide = np.linspace(-90.0, 10.0, V).astype(np.float32)             # masses in every bin and below
+    rng.shuffle(wide)
+    single = np.full(V, -np.inf, dtype=np.float32)                    # one finite logit
+    single[V // 2] = 0.5
+    steps = np.repeat(np.arange(-40.0, 0.0, 2.0), V // 20 + 1)[:V].astype(np.float32)  # bin edges
+    return np.stack([flat, plateau, wide, single, steps])
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("T", [0.05, 1.0, 25.0])
+def test_kept_sets_at_mass_bin_extremes(zb, dtype, T):
+    rng = np.random.default_rng(17)
+    V = 4099
+    x = _shaped_rows(rng, V)
+    if dtype == torch.bfloat16:
+        x = np.where(np.isfinite(x), pen.bf16_round(np.where(np.isfinite(x), x, 0.0)), x)
+    for top_p in (0.3, 0.9, 0.999):
+        rows = x.shape[0]
+        logits, _, _ = _run(zb, x, dtype, [0, rows], T, top_p)
+        got = logits.float().cpu().numpy()
+        for g in range(rows):
+            kept = np.isfinite(got[g])
+            assert np.array_equal(got[g][kept], x[g][kept])
+            assert (got[g][~kept] == -np.inf).all()
+            assert kept.any()
+            assert _kept_ok(x[g].astype(np.float64), kept, T, top_p), (T, top_p, g)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_kept_sets_when_a_mass_bin_outgrows_shared_memory(zb, dtype):
+    """Rows whose boundary bin holds tens of thousands of distinct values (more
+    than the kernel gathers in shared memory): the descent then runs over the
+    row itself."""
+    rng = np.random.default_rng(23)
+    V = 60000
+    band = rng.uniform(0.0, 0.5, V).astype(np.float32)          # one mass octave at T = 1
+    mixed = rng.uniform(-1.0, 1.0, V).astype(np.float32)
+    mixed[rng.choice(V, 50, replace=False)] = 3.0
+    x = np.stack([band, mixed])
+    if dtype == torch.bfloat16:
+        x = pen.bf16_round(x)
+    for T, top_p in ((1.0, 0.5), (1.0, 0.97), (3.0, 0.8)):
+        logits, _, _ = _run(zb, x, dtype, [0, 2], T, top_p)
+        got = logits.float().cpu().numpy()
+        for g in range(2):
+            kept = np.isfinite(got[g])
+            assert np.array_equal(got[g][kept], x[g][kept])
+            assert (got[g][~kept] == -np.inf).all()
+            assert _kept_ok(x[g].astype(np.float64), kept, T, top_p), (T, top_p, g)
