@@ -97,6 +97,30 @@ def test_per_sequence_roofline_of_a_mixed_batch():
     assert e["peak_measured"] == (tf if e["bound"] == "tensor" else hbm_gbs)
 
 
+def test_sustained_tensor_peak_and_the_burst_fraction_beside_it():
+    """Launches timed in long loops are held against the sustained bf16 rate;
+    the entry also gives the fraction against the burst rate, which is lower
+    for a tensor-bound batch (its ideal time is shorter)."""
+    w = wl_make_long()
+    c = bench.algorithmic_counts(w)
+    ideal_s = bench.per_sequence_roofline(w, 6691.1, 1749.2)[0]
+    ideal_b = bench.per_sequence_roofline(w, 6691.1, 1926.3)[0]
+    e = bench.roofline_per_sequence(w, c, attn_ms=ideal_s * 1e3 / 0.7, hbm_peak=6691.1,
+                                    tf_peak=1749.2, peak_src="measured", traffic=None,
+                                    tf_kind="sustained", tf_burst=1926.3)
+    assert e["bound"] == "tensor" and e["peak"] == 1749.2
+    assert e["frac"] == pytest.approx(0.7, abs=1e-4)
+    assert e["frac_of_burst_bf16"] == pytest.approx(0.7 * ideal_b / ideal_s, abs=1e-4)
+    assert e["frac_of_burst_bf16"] < e["frac"]
+    assert "sustained" in e["peak_source"]
+
+
+def wl_make_long():
+    from paper_2609_19868_gb300 import workloads as wl
+
+    return wl.make("long_ctx", small=True).with_mode(0)
+
+
 def test_paged_subset_keeps_each_sequences_attention(oracle_mod):
     """bench's oracle samples of a paged batch keep only the sampled
     sequences' pages, renumbered: their attention must be unchanged."""
