@@ -524,13 +524,14 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
     # k_new, v_new, accept_len, packed in one pinned host buffer) copied to the
     # device, the step, and its output copied back to pinned host memory.
     # The transfers are zarya_copy kernels (a few CTAs moving the bytes through
-    # the pinned buffers' device mapping) on their own streams, pipelined with
-    # the computation over the rotating device buffers (events order each
-    # rotation's copy-in, step and copy-out), as a serving loop would overlap
-    # transfers with compute; the n_rot steps of a rotation cycle, copies
-    # included, are one CUDA graph. (Copy-engine memcpy nodes in the same
-    # graph cost several microseconds per hand-over between a memcpy node and
-    # the kernels around it.)
+    # the pinned buffers' device mapping) or copy-engine memcpys, on their own
+    # streams, pipelined with the computation as a serving loop overlaps
+    # transfers with compute: step i's copy-in runs during step i - 1, its
+    # copy-out during step i + 1. Step i uses rotation i % n_rot; events keep
+    # each rotation's buffers in order (its copy-in waits for the step before
+    # on that rotation to have read them, its step for that step's copy-out to
+    # have read the output). The K steps of a timed region, copies included,
+    # are one CUDA graph.
     def align(x):
         return (x + 255) // 256 * 256
 
@@ -557,15 +558,19 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
     s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
     ev_in = [torch.cuda.Event() for _ in rots]
     ev_done = [torch.cuda.Event() for _ in rots]
+    ev_out = [torch.cuda.Event() for _ in rots]
 
     def e2e_steps(count, engine):
         # stream forks off `stream` and joins back (valid inside a capture);
         # engine: the transfers are copy-engine memcpys instead of zarya_copy
         s_in.wait_stream(stream)
         s_out.wait_stream(stream)
-        for r in range(count):
+        for i in range(count):
+            r = i % n_rot
             db = rots[r]
             with torch.cuda.stream(s_in):
+                if i >= n_rot:
+                    s_in.wait_event(ev_done[r])    # step i - n_rot has read dev_in[r]
                 if engine:
                     dev_in[r].copy_(host_in, non_blocking=True)
                 else:
@@ -573,6 +578,8 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
                 ev_in[r].record(s_in)
             with torch.cuda.stream(stream):
                 stream.wait_event(ev_in[r])
+                if i >= n_rot:
+                    stream.wait_event(ev_out[r])   # its output has been copied out
                 step(db)
                 ev_done[r].record(stream)
             with torch.cuda.stream(s_out):
@@ -581,6 +588,7 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
                     out_h.copy_(db.out, non_blocking=True)
                 else:
                     zb.copy(out_h, db.out, s_out)
+                ev_out[r].record(s_out)
         stream.wait_stream(s_in)
         stream.wait_stream(s_out)
 
@@ -593,10 +601,9 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
         with torch.cuda.stream(stream):
             e2e_steps(n_rot, engine)   # eager warm-up through the public API
         torch.cuda.synchronize()
-        e2e_graph = capture_fn(lambda: e2e_steps(n_rot, engine))
-        e2e_tail = capture_fn(lambda: e2e_steps(tail, engine)) if tail else None
+        e2e_graph = capture_fn(lambda: e2e_steps(K, engine))
         with torch.cuda.stream(stream):
-            for _ in range(max(1, -(-W // n_rot))):
+            for _ in range(max(1, -(-W // K))):
                 e2e_graph.replay()
         torch.cuda.synchronize()
         if world > 1:
@@ -604,10 +611,10 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
 
             dist.barrier()
         with torch.cuda.stream(stream):
-            ms, t0, t1 = timed_reps(region(e2e_graph, e2e_tail), stream, min_reps, min_seconds)
+            ms, t0, t1 = timed_reps(e2e_graph.replay, stream, min_reps, min_seconds)
         sampler_windows.append((entry, "e2e", t0, t1))
         e2e["copy engines" if engine else "zarya_copy kernels"] = rep_stats(ms, K, dev, world)
-        del e2e_graph, e2e_tail
+        del e2e_graph
         assert zb.check_device_error(stream) == 0
     e2e_how = min(e2e, key=lambda k: e2e[k][0])
     res["e2e"] = e2e[e2e_how]
@@ -778,9 +785,10 @@ def run_ours(args):
             "unit": "steps/s",
             "h2d_bytes_per_step": head["h2d"],
             "d2h_bytes_per_step": head["d2h"],
-            "transfers": f"{head['e2e_how']} on side streams pipelined with the steps (one CUDA "
-                         "graph per rotation cycle); the faster of zarya_copy kernels and "
-                         "copy-engine memcpys",
+            "transfers": f"{head['e2e_how']} on side streams pipelined with the steps (step "
+                         "i's copy-in during step i - 1, its copy-out during step i + 1; the K "
+                         "steps and their copies one CUDA graph); the faster of zarya_copy "
+                         "kernels and copy-engine memcpys",
             "steps_per_s_by_transfer": head["e2e_all"],
         },
         "step_forms": {
