@@ -24,8 +24,9 @@
 //
 // Masses are fixed point relative to their bin: a token of bin j adds
 // floor(2^(a + j + 22)) (between 2^21 and 2^22) in units of 2^-(j + 22), and
-// the integer sums are scaled to doubles only for the comparisons, so the
-// boundary does not depend on the order of the GPU's additions (a thread's
+// the decisions compare integer sums in one unit (2^-42 of the maximum's mass;
+// the target ceil(top_p x total) exactly), so the boundary does not depend on
+// the order of the GPU's additions (a thread's
 // slots hold at most 1023 tokens, so 32 bits never overflow). The masses
 // differ from exact ones by the fp32 exponent argument's rounding (below 1e-6
 // relative for any token within 2^20 of the maximum's mass), the approximate
@@ -83,27 +84,54 @@ __device__ __forceinline__ float nuc_ex2(float x) {
   return y;
 }
 
-// 2^-(j + 22) as a double (bin j's unit).
-__device__ __forceinline__ double bin_unit(int j) {
-  return __longlong_as_double(static_cast<long long>(1023 - j - 22) << 52);
+// The decisions compare masses in one fixed-point unit, 2^-42 of the
+// maximum's mass (bin 20's unit): bin j's integer sums scaled by 2^(20 - j),
+// the lighter bins' shifted right (each losing less than one unit). The
+// row's total stays below 2^61 (V < 2^19 tokens of at most 2^42 units).
+constexpr int kCommonBin = 20;
+__device__ __forceinline__ unsigned long long to_common(unsigned long long t, int j) {
+  return j <= kCommonBin ? (t << (kCommonBin - j)) : (t >> (j - kCommonBin));
+}
+
+// ceil(t p) for p in (0, 1) and t < 2^61, exactly: p's 24-bit significand
+// times t in 128 bits, shifted right by p's binary exponent, rounded up.
+__device__ __forceinline__ unsigned long long mul_frac_ceil(unsigned long long t, float p) {
+  const uint32_t u = __float_as_uint(p);
+  const int ex = static_cast<int>((u >> 23) & 0xFFu);
+  const unsigned long long mant = (u & 0x7FFFFFu) | (ex != 0 ? 0x800000u : 0u);
+  const int shift = 150 - (ex != 0 ? ex : 1);   // p = mant 2^-shift, shift >= 24
+  const unsigned long long lo = t * mant, hi = __umul64hi(t, mant);
+  unsigned long long q, rem;
+  if (shift >= 128) {
+    q = 0;
+    rem = lo | hi;
+  } else if (shift >= 64) {
+    q = hi >> (shift - 64);
+    rem = lo | (hi & ((1ull << (shift - 64)) - 1ull));
+  } else {
+    q = (lo >> shift) | (hi << (64 - shift));
+    rem = lo & ((1ull << shift) - 1ull);
+  }
+  return q + (rem != 0ull ? 1ull : 0ull);
 }
 
 // A token's mass in its bin's units, and its bin. The same arithmetic decides
-// the bins in stage 1, in the key-range search and in stage 2.
+// the bins in stage 1, in the key-range search and in stage 2. The mass is
+// floor(e 2^(j + 22)) for e = 2^c: the product is exact (a power of two), and
+// adding 2^23 with rounding toward zero leaves floor(v) in the low bits (v is
+// below 2^23), so the sum's bits minus 2^23's are the integer mass.
 struct Mass {
   uint32_t q;   // 0 for a massless token (a <= -42, or NaN)
   uint32_t j;
 };
 __device__ __forceinline__ Mass token_mass(float x, float k2, float neg_mk) {
   const float a = fmaf(x, k2, neg_mk);
-  const float c = fminf(fmaxf(a, kMassFloorUp), 0.f);
-  const uint32_t j = __float_as_uint(__fmaf_rz(c, -1.f, kBinMagic)) - kBinMagicBits;
-  // e = 2^c lies in [2^-(j+1), 2^-j] up to the approximation: its 24-bit
-  // significand shifted to the units of 2^-(j + 22)
-  const uint32_t u = __float_as_uint(nuc_ex2(c));
-  const uint32_t r = min(128u - (u >> 23) - j, 31u);
-  const uint32_t q = ((u & 0x7FFFFFu) | 0x800000u) >> r;
-  return Mass{a > kMassFloor ? q : 0u, j};
+  const float c = a > kMassFloor ? fminf(a, 0.f) : -INFINITY;   // -inf: e = 0
+  const uint32_t j =
+      __float_as_uint(__fmaf_rz(fmaxf(c, kMassFloorUp), -1.f, kBinMagic)) - kBinMagicBits;
+  const float scale = __uint_as_float((j + 149u) << 23);   // 2^(j + 22)
+  const float v = nuc_ex2(c) * scale;
+  return Mass{__float_as_uint(__fadd_rz(v, 8388608.f)) - 0x4B000000u, j};
 }
 
 // The bin of a logit (kMassBins for a massless one): token_mass's bin test.
@@ -194,7 +222,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   __shared__ int s_seg[kNucWarps];
   __shared__ int s_pick, s_over;
   __shared__ uint32_t s_klo, s_khi, s_prefix;
-  __shared__ double s_above, s_target;
+  __shared__ unsigned long long s_above, s_target;
   grid_dependency_wait();
   grid_launch_dependents();
   const int g = blockIdx.x;
@@ -252,17 +280,17 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   }
   __syncthreads();
   if (tid == 0) {
-    double tot = 0.0;
+    unsigned long long tot = 0;
 #pragma unroll 1
-    for (int j = 0; j < kMassBins; ++j) tot += static_cast<double>(bins[j]) * bin_unit(j);
-    const double target = static_cast<double>(a.top_p) * tot;
+    for (int j = 0; j < kMassBins; ++j) tot += to_common(bins[j], j);
+    const unsigned long long target = tot > 0 ? mul_frac_ceil(tot, a.top_p) : 0ull;
     int pick = -1, lowest = -1;
-    double cum = 0.0;
-    if (tot > 0.0) {
+    unsigned long long cum = 0;
+    if (tot > 0) {
 #pragma unroll 1
       for (int j = 0; j < kMassBins; ++j) {
         if (bins[j] == 0ull) continue;
-        const double h = static_cast<double>(bins[j]) * bin_unit(j);
+        const unsigned long long h = to_common(bins[j], j);
         lowest = j;
         if (cum + h >= target) {
           pick = j;
@@ -270,11 +298,11 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
         }
         cum += h;
       }
-      if (pick < 0) {   // the target is beyond the mass (rounding): keep down to the lowest bin
+      if (pick < 0) {   // the target is beyond the mass (truncation): keep down to the lowest bin
         pick = lowest;
-        cum = 0.0;
+        cum = 0;
 #pragma unroll 1
-        for (int j = 0; j < pick; ++j) cum += static_cast<double>(bins[j]) * bin_unit(j);
+        for (int j = 0; j < pick; ++j) cum += to_common(bins[j], j);
       }
     }
     s_pick = pick;
@@ -304,22 +332,55 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   const uint32_t klo = s_klo, range = s_khi - s_klo;
   uint32_t prefix = 0;   // the key offset of x* above the current level
   if (range > 0) {
-    // Gather the keys of the bin into this warp's segment. The loop runs the
-    // same number of times in every lane of the warp (ballots need all 32).
+    // Gather the keys of the bin into this warp's segment. Each lane marks its
+    // logits in [x(klo), x(khi)] (a float test that takes every key of the
+    // range; a signed zero it takes beside them fails the descent's key test)
+    // in a bit mask per vector, and a warp prefix sum of the counts places
+    // them. The loop runs the same number of times in every lane of the warp
+    // (the shuffles need all 32).
     TBits* seg = reinterpret_cast<TBits*>(reinterpret_cast<unsigned char*>(smem) + kDigitBytes) +
                  warp * kSegKeys;
-    int cnt = 0;
-    auto gather = [&](uint32_t f, bool valid) {
-      const uint32_t key = logit_key<kKeyBits>(f);
-      const bool in = valid && key - klo <= range;
-      const unsigned bal = __ballot_sync(0xffffffffu, in);
-      const int pos = cnt + __popc(bal & ((1u << lane) - 1u));
-      if (in && pos < kSegKeys) seg[pos] = static_cast<TBits>(key);
-      cnt += __popc(bal);
+    int cnt = 0;   // keys this warp found (uniform over the warp)
+    const uint32_t flo = key_bits<kKeyBits>(klo), fhi = key_bits<kKeyBits>(s_khi);
+    // bit e set: logit e of the vector is in the range
+    auto in_bits = [&](const uint4& v) -> uint32_t {
+      if constexpr (sizeof(TBits) == 2) {
+        const uint32_t lo2 = (flo >> 16) | (flo & 0xFFFF0000u), hi2 = (fhi >> 16) | (fhi & 0xFFFF0000u);
+        const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&lo2);
+        const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&hi2);
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+        uint32_t x = 0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          x |= ((__hge2_mask(h[k], lo) & __hle2_mask(h[k], hi)) & 0x00010001u) << (2 * k);
+        return (x | (x >> 15)) & 0xFFu;
+      } else {
+        const float lo = __uint_as_float(flo), hi = __uint_as_float(fhi);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        uint32_t x = 0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float f = __uint_as_float(w[k]);
+          x |= static_cast<uint32_t>(f >= lo && f <= hi) << k;
+        }
+        return x;
+      }
+    };
+    // the fp32 bits of logit e of a vector
+    auto logit_bits = [&](const uint4& v, int e) -> uint32_t {
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      if constexpr (sizeof(TBits) == 2) {
+        const uint32_t x = w[e >> 1];
+        return (e & 1) ? (x & 0xFFFF0000u) : (x << 16);
+      } else {
+        return w[e];
+      }
     };
     const int warp0 = tid - lane;
     for (int i0 = warp0; i0 < nvec; i0 += kNucUnroll * kNucThreads) {
       uint4 w[kNucUnroll];
+      uint32_t bits[kNucUnroll];
+      int c = 0;
 #pragma unroll
       for (int u = 0; u < kNucUnroll; ++u) {
         const int i = i0 + u * kNucThreads + lane;
@@ -327,13 +388,33 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
       }
 #pragma unroll
       for (int u = 0; u < kNucUnroll; ++u) {
-        const bool valid = i0 + u * kNucThreads + lane < nvec;
-        each_logit<TBits>(w[u], [&](uint32_t f) { gather(f, valid); });
+        bits[u] = i0 + u * kNucThreads + lane < nvec ? in_bits(w[u]) : 0u;
+        c += __popc(bits[u]);
       }
+      int incl = c;   // inclusive prefix sum of the lanes' counts
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += t;
+      }
+      int pos = cnt + incl - c;
+#pragma unroll
+      for (int u = 0; u < kNucUnroll; ++u) {
+        for (uint32_t m = bits[u]; m != 0u; m &= m - 1u, ++pos) {
+          const int e = __ffs(m) - 1;
+          if (pos < kSegKeys) seg[pos] = static_cast<TBits>(logit_key<kKeyBits>(logit_bits(w[u], e)));
+        }
+      }
+      cnt += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (warp == 0) {   // the scalar tail (fewer than kPerVec logits)
       const bool valid = tail0 + lane < V;
-      gather(valid ? widen(row[tail0 + lane]) : 0u, valid);
+      const uint32_t key = valid ? logit_key<kKeyBits>(widen(row[tail0 + lane])) : 0u;
+      const bool in = valid && key - klo <= range;
+      const unsigned bal = __ballot_sync(0xffffffffu, in);
+      const int p = cnt + __popc(bal & ((1u << lane) - 1u));
+      if (in && p < kSegKeys) seg[p] = static_cast<TBits>(key);
+      cnt += __popc(bal);
     }
     if (lane == 0) {
       s_seg[warp] = min(cnt, kSegKeys);
@@ -347,8 +428,8 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
     // over the gathered keys (or the row, when a segment overflowed).
     const int nbits = 32 - __clz(range);
     const int levels = (nbits + kDigitBits - 1) / kDigitBits;
-    const double unit = bin_unit(jbin), target = s_target;
-    double above = s_above;   // mass of the tokens above the current range
+    const unsigned long long target = s_target;
+    unsigned long long above = s_above;   // mass of the tokens above the current range
     for (int level = 0; level < levels; ++level) {
       const int shift = kDigitBits * (levels - 1 - level);
 #pragma unroll
@@ -378,12 +459,12 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
       }
       __syncthreads();
       if (tid == 0) {
-        double cum = above;
+        unsigned long long cum = above;
         int pick = -1, lowest = -1;
 #pragma unroll 1
         for (int k = kDigits - 1; k >= 0; --k) {
           if (bins[k] == 0ull) continue;
-          const double h = static_cast<double>(bins[k]) * unit;
+          const unsigned long long h = to_common(bins[k], jbin);
           lowest = k;
           if (cum + h >= target) {
             pick = k;
@@ -391,11 +472,11 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
           }
           cum += h;
         }
-        if (pick < 0) {   // the target is beyond the mass (rounding): keep down to the lowest digit
+        if (pick < 0) {   // the target is beyond the mass (truncation): keep down to the lowest digit
           pick = lowest < 0 ? 0 : lowest;
           cum = above;
 #pragma unroll 1
-          for (int k = kDigits - 1; k > pick; --k) cum += static_cast<double>(bins[k]) * unit;
+          for (int k = kDigits - 1; k > pick; --k) cum += to_common(bins[k], jbin);
         }
         s_prefix = (prefix << kDigitBits) | static_cast<uint32_t>(pick);
         s_above = cum;
@@ -406,31 +487,43 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
     }
   }
 
-  // x*'s key is klo + prefix: every logit below it becomes -inf
-  const uint32_t xkey = klo + prefix;
+  // x* is the logit of key klo + prefix: every logit below it becomes -inf
+  // (a float comparison: a signed zero equal to x* is kept, and NaN logits
+  // stay in place)
+  const uint32_t xbits = key_bits<kKeyBits>(klo + prefix);
   uint4* wrow4 = reinterpret_cast<uint4*>(row);
-  for_each_vec(row4, nvec, tid, [&](const uint4& v, int i) {
-    uint32_t w[4] = {v.x, v.y, v.z, v.w};
-    bool cut = false;
+  if constexpr (sizeof(TBits) == 2) {
+    const uint32_t x2 = (xbits >> 16) | (xbits & 0xFFFF0000u);
+    const __nv_bfloat162 xs = *reinterpret_cast<const __nv_bfloat162*>(&x2);
+    for_each_vec(row4, nvec, tid, [&](const uint4& v, int i) {
+      uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t any = 0;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      if constexpr (sizeof(TBits) == 2) {
-        const bool cl = logit_key<16>(w[k] << 16) < xkey;
-        const bool ch = logit_key<16>(w[k] & 0xFFFF0000u) < xkey;
-        w[k] = (cl ? 0xFF80u : (w[k] & 0xFFFFu)) | (ch ? 0xFF800000u : (w[k] & 0xFFFF0000u));
-        cut = cut || cl || ch;
-      } else {
-        const bool c = logit_key<32>(w[k]) < xkey;
-        w[k] = c ? 0xFF800000u : w[k];
-        cut = cut || c;
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t cut = __hlt2_mask(*reinterpret_cast<const __nv_bfloat162*>(&w[k]), xs);
+        w[k] = (w[k] & ~cut) | (0xFF80FF80u & cut);
+        any |= cut;
       }
-    }
-    if (cut) wrow4[i] = make_uint4(w[0], w[1], w[2], w[3]);
-  });
+      if (any) wrow4[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    });
+  } else {
+    const float xs = __uint_as_float(xbits);
+    for_each_vec(row4, nvec, tid, [&](const uint4& v, int i) {
+      uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      bool any = false;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const bool cut = __uint_as_float(w[k]) < xs;
+        w[k] = cut ? 0xFF800000u : w[k];
+        any = any || cut;
+      }
+      if (any) wrow4[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    });
+  }
   const TBits neg_inf = sizeof(TBits) == 2 ? static_cast<TBits>(0xFF80u)
                                            : static_cast<TBits>(0xFF800000u);
   for (int v = tail0 + tid; v < V; v += kNucThreads)
-    if (logit_key<kKeyBits>(widen(row[v])) < xkey) row[v] = neg_inf;
+    if (__uint_as_float(widen(row[v])) < __uint_as_float(xbits)) row[v] = neg_inf;
 }
 
 }  // namespace
