@@ -509,7 +509,8 @@ zarya_status zarya_repetition_penalty(void* logits, const int32_t* hist_offsets,
  * exact arithmetic only where the mass at a boundary lies within about 1e-6 of
  * top_p.
  *  logits   [desc->total_rows, desc->row_stride] of desc->dtype (read and
- *           written; 16-byte aligned); rows of no sequence are untouched
+ *           written; 16-byte aligned); rows of no sequence are untouched,
+ *           and NaN logits are left in place (they carry no mass)
  *  top_p    in (0, 1); top_p >= 1 returns at once (nothing to cut)
  * desc supplies batch, vocab, dtype, total_rows, row_stride, row_offsets and
  * temperature; its other fields are checked as for zarya_draft_select.

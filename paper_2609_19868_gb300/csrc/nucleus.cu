@@ -16,18 +16,21 @@
 // range of order-preserving logit keys (sign-flipped bits; 16 bits for bf16,
 // 32 for fp32) by a 32-way search over the monotone bin function, a pass over
 // the row gathers the keys in that range into shared memory (each warp its
-// own segment, placed by ballots), and stage 2 runs a radix descent over them,
-// 4 bits of the key offset per level, again with private slots per thread: a
-// level sums each candidate's mass into its digit, and the digit where the
-// mass counted from the top reaches top_p is fixed. A row whose bin holds more
-// keys than the shared memory takes the descent's levels over the row instead.
+// own segment, placed by a warp prefix sum of the lanes' counts), and stage 2
+// runs a radix descent over them, 4 bits of the key offset per level, again
+// with private slots per thread: a level sums each candidate's mass into its
+// digit, and the digit where the mass counted from the top reaches top_p is
+// fixed. A row whose bin holds more keys than the shared memory takes the
+// descent's levels over the row instead. The last pass cuts every logit
+// below x* (a float comparison, so a signed zero equal to x* stays, and NaN
+// logits are left in place).
 //
 // Masses are fixed point relative to their bin: a token of bin j adds
 // floor(2^(a + j + 22)) (between 2^21 and 2^22) in units of 2^-(j + 22), and
 // the decisions compare integer sums in one unit (2^-42 of the maximum's mass;
 // the target ceil(top_p x total) exactly), so the boundary does not depend on
-// the order of the GPU's additions (a thread's
-// slots hold at most 1023 tokens, so 32 bits never overflow). The masses
+// the order of the GPU's additions (a thread's slots hold at most 1023
+// tokens, so 32 bits never overflow). The masses
 // differ from exact ones by the fp32 exponent argument's rounding (below 1e-6
 // relative for any token within 2^20 of the maximum's mass), the approximate
 // exp2 (2^-22) and the truncation (below 2^-21 relative; tokens under 2^-42 of

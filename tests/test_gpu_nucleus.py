@@ -187,3 +187,23 @@ def test_kept_sets_when_a_mass_bin_outgrows_shared_memory(zb, dtype):
             assert np.array_equal(got[g][kept], x[g][kept])
             assert (got[g][~kept] == -np.inf).all()
             assert _kept_ok(x[g].astype(np.float64), kept, T, top_p), (T, top_p, g)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_signed_zeros_at_the_boundary_are_kept_together(zb, dtype):
+    """x* = 0 with +0.0 and -0.0 logits both present: the kept set is
+    {x >= x*}, so both zeros stay (they are equal values)."""
+    V = 64
+    x = np.full(V, -6.0, dtype=np.float32)
+    x[:4] = 1.0
+    x[4:14] = 0.0
+    x[14:24] = -0.0
+    rows = np.stack([x, x[::-1].copy()])
+    for top_p in (0.5, 0.8):
+        logits, _, _ = _run(zb, rows, dtype, [0, 2], 1.0, top_p)
+        got = logits.float().cpu().numpy()
+        for g in range(2):
+            kept = np.isfinite(got[g])
+            zeros = rows[g] == 0.0
+            assert kept[zeros].all() or not kept[zeros].any(), "the zeros split"
+            assert _kept_ok(rows[g].astype(np.float64), kept, 1.0, top_p), (top_p, g)
