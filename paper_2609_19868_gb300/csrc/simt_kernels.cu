@@ -76,27 +76,33 @@ __device__ __forceinline__ long long token_row(const int32_t* page_table, int pa
 
 constexpr int kF32Warps = 8;   // warps per CTA of the fp32 attention kernel
 
+// One CTA per (sequence, head, block row). The row's visible keys (the
+// earlier slots' hidden block rows [P, hide_hi) skipped) go in chunks of 32 to
+// the CTA's warps in turn; within a chunk lane k scores key k with a whole
+// dot product, the warp takes the chunk's maximum and sum and broadcasts the
+// weights to accumulate O (lane l holds columns l, l + 32, ...), an online
+// softmax over the warp's chunks. The warps' partial (m, l, O) then merge in
+// shared memory: O = sum_w e^(m_w - M) O_w / sum_w e^(m_w - M) l_w.
 template <int kPerLane>
 __global__ void __launch_bounds__(kF32Warps * 32)
 slot_attn_f32_kernel(const SimtParams p) {
   grid_dependency_wait();
   grid_launch_dependents();
   constexpr int D = kPerLane * 32;
-  const int lane = threadIdx.x & 31;
-  const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const long long per_b = static_cast<long long>(p.Hq) * p.max_rows;
-  const int b = static_cast<int>(wid / per_b);
+  const int b = static_cast<int>(blockIdx.x / per_b);
   if (b >= p.B) return;
-  const int rem = static_cast<int>(wid - b * per_b);
+  const int rem = static_cast<int>(blockIdx.x - b * per_b);
   const int h = rem / p.max_rows;
   const int r = rem - h * p.max_rows;
   int P, R, mode, row0;
   const int code = check_sequence(p, b, &P, &R, &mode, &row0);
   if (code != 0) {
-    if (h == 0 && r == 0 && lane == 0) record_error(p.err, code);
+    if (h == 0 && r == 0 && threadIdx.x == 0) record_error(p.err, code);
     return;
   }
-  if (r >= R) return;
+  if (r >= R) return;   // uniform over the CTA
   const int g = p.Hq / p.Hkv;
   const int j = h / g;
   const int n_vis = (mode == ZARYA_MASK_BIDIR_BLOCK) ? P + R : P + r + 1;
@@ -106,23 +112,19 @@ slot_attn_f32_kernel(const SimtParams p) {
                    (static_cast<long long>(row0 + r) * p.Hq + h) * D;
   const float* kc = reinterpret_cast<const float*>(p.k_cache);
   const float* vc = reinterpret_cast<const float*>(p.v_cache);
-  // This warp's query row in shared memory (every lane reads all of it).
-  __shared__ float4 qs[kF32Warps][D / 4];
-  float* qw = reinterpret_cast<float*>(qs[threadIdx.x >> 5]);
-#pragma unroll
-  for (int x = 0; x < kPerLane; ++x) qw[lane + 32 * x] = q[lane + 32 * x];
-  __syncwarp();
-  // Online softmax over chunks of 32 visible keys (the earlier slots' hidden
-  // block rows [P, hide_hi) skipped): lane k scores key k of the chunk with a
-  // whole dot product, the warp takes the chunk's maximum and sum, and the
-  // chunk's weights are broadcast to accumulate O, lane l holding columns
-  // l, l + 32, ...
+  __shared__ float4 qs[D / 4];                 // the query row (every lane reads all of it)
+  __shared__ float s_o[kF32Warps][D];          // the warps' partial outputs
+  __shared__ float s_m[kF32Warps], s_l[kF32Warps];
+  __shared__ int s_bad;
+  if (threadIdx.x == 0) s_bad = 0;
+  for (int i = threadIdx.x; i < D; i += kF32Warps * 32) reinterpret_cast<float*>(qs)[i] = q[i];
+  __syncthreads();
   const int nv = P + (n_vis - hide_hi);
   float o[kPerLane];
 #pragma unroll
   for (int x = 0; x < kPerLane; ++x) o[x] = 0.f;
   float m = -INFINITY, l = 0.f;
-  for (int base = 0; base < nv; base += 32) {
+  for (int base = warp * 32; base < nv; base += kF32Warps * 32) {
     const int i = base + lane;
     float s = -INFINITY;
     long long row = 0;   // first element of this lane's key row (K and V)
@@ -140,7 +142,7 @@ slot_attn_f32_kernel(const SimtParams p) {
 #pragma unroll 8
         for (int d = 0; d < D / 4; ++d) {
           const float4 kv = k4[d];
-          const float4 qv = qs[threadIdx.x >> 5][d];
+          const float4 qv = qs[d];
           dot0 = fmaf(qv.x, kv.x, dot0);
           dot1 = fmaf(qv.y, kv.y, dot1);
           dot0 = fmaf(qv.z, kv.z, dot0);
@@ -150,8 +152,8 @@ slot_attn_f32_kernel(const SimtParams p) {
       }
     }
     if (__any_sync(0xffffffffu, bad)) {
-      if (lane == 0) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
-      return;
+      if (lane == 0) s_bad = 1;
+      break;
     }
     float cm = s;
 #pragma unroll
@@ -177,9 +179,34 @@ slot_attn_f32_kernel(const SimtParams p) {
     }
     m = m_new;
   }
-  float* out = reinterpret_cast<float*>(p.out) + (static_cast<long long>(row0 + r) * p.Hq + h) * D;
+  if (lane == 0) {
+    s_m[warp] = m;
+    s_l[warp] = l;
+  }
 #pragma unroll
-  for (int x = 0; x < kPerLane; ++x) out[lane + 32 * x] = o[x] / l;
+  for (int x = 0; x < kPerLane; ++x) s_o[warp][lane + 32 * x] = o[x];
+  __syncthreads();
+  if (s_bad) {
+    if (threadIdx.x == 0) record_error(p.err, ZARYA_DEVERR_PAGE_ID);
+    return;
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kF32Warps; ++w) M = fmaxf(M, s_m[w]);
+  float L = 0.f;
+  float wt[kF32Warps];
+#pragma unroll
+  for (int w = 0; w < kF32Warps; ++w) {
+    wt[w] = (s_m[w] == -INFINITY) ? 0.f : expf(s_m[w] - M);
+    L = fmaf(wt[w], s_l[w], L);
+  }
+  float* out = reinterpret_cast<float*>(p.out) + (static_cast<long long>(row0 + r) * p.Hq + h) * D;
+  for (int t = threadIdx.x; t < D; t += kF32Warps * 32) {
+    float acc = 0.f;
+#pragma unroll
+    for (int w = 0; w < kF32Warps; ++w) acc = fmaf(wt[w], s_o[w][t], acc);
+    out[t] = acc / L;
+  }
 }
 
 // At most this many CTAs share one sequence's rows, so that a commit can
@@ -296,12 +323,9 @@ cudaError_t launch_commit_lens(const AppendParams& p, cudaStream_t stream) {
 }
 
 cudaError_t launch_slot_attn_f32(const SimtParams& p, cudaStream_t stream) {
-  const long long warps = static_cast<long long>(p.B) * p.Hq * p.max_rows;
-  const long long threads = warps * 32;
-  const int block = 256;
-  const long long grid = (threads + block - 1) / block;
+  const long long grid = static_cast<long long>(p.B) * p.Hq * p.max_rows;   // one CTA per row
   if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  PdlLaunch l(dim3(static_cast<unsigned>(grid)), dim3(block), 0, stream);
+  PdlLaunch l(dim3(static_cast<unsigned>(grid)), dim3(kF32Warps * 32), 0, stream);
   switch (p.D / 32) {
     case 1: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<1>, p);
     case 2: return cudaLaunchKernelEx(&l.cfg, slot_attn_f32_kernel<2>, p);
