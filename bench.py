@@ -616,6 +616,10 @@ def measure_workload(entry, args, dev, stream, world, rank, K, W, min_reps, min_
         e2e["copy engines" if engine else "zarya_copy kernels"] = rep_stats(ms, K, dev, world)
         del e2e_graph
         assert zb.check_device_error(stream) == 0
+        # every step computes the same output (a stationary workload): what
+        # the last copy-out left in pinned memory is the device's result
+        assert torch.equal(out_h.view(torch.uint8), rots[(K - 1) % n_rot].out.cpu().view(torch.uint8)), \
+            "end-to-end output differs from the device result"
     e2e_how = min(e2e, key=lambda k: e2e[k][0])
     res["e2e"] = e2e[e2e_how]
 
