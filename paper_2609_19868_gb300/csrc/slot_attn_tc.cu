@@ -106,6 +106,30 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// The softmax numerators of one row over 64 score columns, s[c] → 2^(s[c] *
+// sl2 - m), packed as 32 bf16 pairs into pk; returns their fp32 sum.  The
+// exponent arguments and the four running sums use the paired fp32
+// instructions.  Each half rounds exactly as the scalar fmaf / add would, so
+// the result is the scalar loop's bit for bit, with half the issue slots.
+__device__ __forceinline__ float exp_pack_row(const float* s, float sl2, float m,
+                                              float pk[32]) {
+  const float2 k = make_float2(sl2, sl2), nm = make_float2(-m, -m);
+  float2 r01 = make_float2(0.f, 0.f), r23 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int x = 0; x < 32; x += 2) {
+    const int c = 2 * x;
+    const float2 a01 = __ffma2_rn(make_float2(s[c + 0], s[c + 1]), k, nm);
+    const float2 a23 = __ffma2_rn(make_float2(s[c + 2], s[c + 3]), k, nm);
+    const float2 e01 = make_float2(fast_exp2(a01.x), fast_exp2(a01.y));
+    const float2 e23 = make_float2(fast_exp2(a23.x), fast_exp2(a23.y));
+    r01 = __fadd2_rn(r01, e01);
+    r23 = __fadd2_rn(r23, e23);
+    pk[x] = __uint_as_float(pack_bf16(e01.x, e01.y));
+    pk[x + 1] = __uint_as_float(pack_bf16(e23.x, e23.y));
+  }
+  return (r01.x + r01.y) + (r23.x + r23.y);
+}
+
 __device__ __forceinline__ void named_bar_sync(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
@@ -835,23 +859,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
       // P = 2^(s * scale * log2 e - m) as packed bf16 pairs over the first 32
       // columns of this group's half of the S buffer (S is in registers).
       float pk[32];
-      float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
-#pragma unroll
-      for (int x = 0; x < 32; x += 2) {
-        const int c = 2 * x;
-        const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
-        const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
-        const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
-        const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
-        rs0 += e0;
-        rs1 += e1;
-        rs2 += e2;
-        rs3 += e3;
-        pk[x] = __uint_as_float(pack_bf16(e0, e1));
-        pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
-      }
+      l_run += exp_pack_row(s, sl2, m_use, pk);
       tmem_st_32x32b_x32(t_s, pk);
-      l_run += (rs0 + rs1) + (rs2 + rs3);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->p_full[sb]);
@@ -1438,23 +1447,8 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
       // P = 2^(s * scale * log2 e - m) for this group's keys, packed bf16
       // pairs over the first 32 columns of its half of S.
       float pk[32];
-      float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
-#pragma unroll
-      for (int x = 0; x < 32; x += 2) {
-        const int c = 2 * x;
-        const float e0 = fast_exp2(fmaf(s[c + 0], sl2, -m_use));
-        const float e1 = fast_exp2(fmaf(s[c + 1], sl2, -m_use));
-        const float e2 = fast_exp2(fmaf(s[c + 2], sl2, -m_use));
-        const float e3 = fast_exp2(fmaf(s[c + 3], sl2, -m_use));
-        rs0 += e0;
-        rs1 += e1;
-        rs2 += e2;
-        rs3 += e3;
-        pk[x] = __uint_as_float(pack_bf16(e0, e1));
-        pk[x + 1] = __uint_as_float(pack_bf16(e2, e3));
-      }
+      l_run += exp_pack_row(s, sl2, m_use, pk);
       tmem_st_32x32b_x32(t_s + grp * 64, pk);
-      l_run += (rs0 + rs1) + (rs2 + rs3);
       if (t) {
         m_runB = m_run;
         l_runB = l_run;
