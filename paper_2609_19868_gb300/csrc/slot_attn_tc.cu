@@ -106,6 +106,26 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// max(a, b, c) in one instruction (the three-input form of max.f32).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Row maximum of 64 scores: four chains of sixteen, 34 max instructions.
+__device__ __forceinline__ float max64(const float (&s)[64]) {
+  float m4[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    float a = fmax3(s[k], s[k + 4], s[k + 8]);
+#pragma unroll
+    for (int x = 12; x < 60; x += 8) a = fmax3(a, s[x + k], s[x + 4 + k]);
+    m4[k] = fmaxf(a, s[60 + k]);
+  }
+  return fmax3(fmaxf(m4[0], m4[1]), m4[2], m4[3]);
+}
+
 // The softmax numerators of one row over 64 score columns, s[c] → 2^(s[c] *
 // sl2 - m), packed as 32 bf16 pairs into pk; returns their fp32 sum.  The
 // exponent arguments and the four running sums use the paired fp32
@@ -800,16 +820,7 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
         for (int x = 0; x < 64; ++x)
           if (c0 + x >= P && c0 + x < hide_hi) s[x] = -INFINITY;
       }
-      float mx[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) mx[k] = s[k];
-#pragma unroll
-      for (int x = 8; x < 64; x += 8)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], s[x + k]);
-      const float mt4 = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-      const float mt8 = fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]));
-      const float m_new = fmaxf(m_run, fmaxf(mt4, mt8) * sl2);
+      const float m_new = fmaxf(m_run, max64(s) * sl2);
       const bool need = m_new > m_run + 8.0f;
       const bool warp_need = __any_sync(0xffffffffu, need);
       float alpha = 1.f;
@@ -1113,19 +1124,6 @@ struct PairBars {
 
 constexpr uint32_t kPairSmemBytes = kPOffBar + ((sizeof(PairBars) + 127) / 128) * 128 + 1024;
 static_assert(kPairSmemBytes <= 232448, "shared memory budget (paired M-tiles)");
-
-// Row maximum of 64 scores.
-__device__ __forceinline__ float max64(const float (&s)[64]) {
-  float m8[8];
-#pragma unroll
-  for (int k = 0; k < 8; ++k) m8[k] = s[k];
-#pragma unroll
-  for (int x = 8; x < 64; x += 8)
-#pragma unroll
-    for (int k = 0; k < 8; ++k) m8[k] = fmaxf(m8[k], s[x + k]);
-  return fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-               fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-}
 
 __global__ void __launch_bounds__(kThreads, 1)
 slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
