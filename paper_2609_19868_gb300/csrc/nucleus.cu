@@ -137,6 +137,26 @@ __device__ __forceinline__ Mass token_mass(float x, float k2, float neg_mk) {
   return Mass{__float_as_uint(__fadd_rz(v, 8388608.f)) - 0x4B000000u, j};
 }
 
+// token_mass for two logits at once: the same operations, the ones with a
+// paired fp32 form taken two at a time (each half rounds exactly as the
+// scalar instruction does), so each result is token_mass's bit for bit.
+__device__ __forceinline__ void token_mass2(float x0, float x1, float k2, float neg_mk, Mass& s0,
+                                            Mass& s1) {
+  const float2 a = __ffma2_rn(make_float2(x0, x1), make_float2(k2, k2), make_float2(neg_mk, neg_mk));
+  const float c0 = a.x > kMassFloor ? fminf(a.x, 0.f) : -INFINITY;
+  const float c1 = a.y > kMassFloor ? fminf(a.y, 0.f) : -INFINITY;
+  const float2 y = __ffma2_rz(make_float2(fmaxf(c0, kMassFloorUp), fmaxf(c1, kMassFloorUp)),
+                              make_float2(-1.f, -1.f), make_float2(kBinMagic, kBinMagic));
+  s0.j = __float_as_uint(y.x) - kBinMagicBits;
+  s1.j = __float_as_uint(y.y) - kBinMagicBits;
+  const float2 scale = make_float2(__uint_as_float((s0.j + 149u) << 23),
+                                   __uint_as_float((s1.j + 149u) << 23));
+  const float2 v = __fmul2_rn(make_float2(nuc_ex2(c0), nuc_ex2(c1)), scale);
+  const float2 r = __fadd2_rz(v, make_float2(8388608.f, 8388608.f));
+  s0.q = __float_as_uint(r.x) - 0x4B000000u;
+  s1.q = __float_as_uint(r.y) - 0x4B000000u;
+}
+
 // The bin of a logit (kMassBins for a massless one): token_mass's bin test.
 __device__ __forceinline__ int token_bin(float x, float k2, float neg_mk) {
   const float a = fmaf(x, k2, neg_mk);
@@ -156,6 +176,19 @@ template <int kKeyBits>
 __device__ __forceinline__ uint32_t key_bits(uint32_t key) {
   const uint32_t k = key << (32 - kKeyBits);
   return (k & 0x80000000u) ? (k ^ 0x80000000u) : ~k & (0xFFFFFFFFu << (32 - kKeyBits));
+}
+
+// Calls f(fp32 bits, fp32 bits) for each pair of logits of a 16-byte vector.
+template <typename TBits, typename F>
+__device__ __forceinline__ void each_logit_pair(const uint4& v, F&& f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if (sizeof(TBits) == 2) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) f(w[k] << 16, w[k] & 0xFFFF0000u);
+  } else {
+    f(w[0], w[1]);
+    f(w[2], w[3]);
+  }
 }
 
 // Calls f(fp32 bits) for each logit of a 16-byte vector.
@@ -263,16 +296,23 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   if (!(m > -INFINITY)) return;   // every logit -inf (or NaN): nothing to cut
   const float k2 = a.k2, neg_mk = -m * a.k2;
 
-  // Stage 1: the mass bins in private slots.
+  // Stage 1: the mass bins in private slots. A slot has one writer, so its
+  // updates are shared-memory reductions (no load-add-store chain from one
+  // logit to the next, and integer sums do not depend on their order).
   uint32_t* own = smem + tid;
 #pragma unroll
   for (int j = 0; j < kMassBins; ++j) own[j * kNucThreads] = 0u;
-  auto add_mass = [&](uint32_t f) {
-    const Mass s = token_mass(__uint_as_float(f), k2, neg_mk);
-    own[s.j * kNucThreads] += s.q;
+  auto add_mass2 = [&](uint32_t f0, uint32_t f1) {
+    Mass s0, s1;
+    token_mass2(__uint_as_float(f0), __uint_as_float(f1), k2, neg_mk, s0, s1);
+    atomicAdd(own + s0.j * kNucThreads, s0.q);
+    atomicAdd(own + s1.j * kNucThreads, s1.q);
   };
-  for_each_vec(row4, nvec, tid, [&](const uint4& v, int) { each_logit<TBits>(v, add_mass); });
-  for (int v = tail0 + tid; v < V; v += kNucThreads) add_mass(widen(row[v]));
+  for_each_vec(row4, nvec, tid, [&](const uint4& v, int) { each_logit_pair<TBits>(v, add_mass2); });
+  for (int v = tail0 + tid; v < V; v += kNucThreads) {
+    const Mass s = token_mass(__uint_as_float(widen(row[v])), k2, neg_mk);
+    atomicAdd(own + s.j * kNucThreads, s.q);
+  }
   __syncthreads();
   for (int j = warp; j < kMassBins; j += kNucWarps) {   // fixed summation order
     unsigned long long t = 0;
@@ -442,7 +482,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
         if (d > range) return;
         if (level > 0 && (d >> (shift + kDigitBits)) != prefix) return;
         const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk);
-        own[((d >> shift) & (kDigits - 1)) * kNucThreads] += s.q;
+        atomicAdd(own + ((d >> shift) & (kDigits - 1)) * kNucThreads, s.q);
       };
       if (!over) {
         for (int e = lane; e < n_mine; e += 32) add(seg[e]);
