@@ -71,6 +71,11 @@ constexpr int kDigits = 1 << kDigitBits;
 constexpr size_t kNucSmem = static_cast<size_t>(kMassBins) * kNucThreads * sizeof(uint32_t);
 constexpr size_t kDigitBytes = static_cast<size_t>(kDigits) * kNucThreads * sizeof(uint32_t);
 constexpr size_t kCandBytes = kNucSmem - kDigitBytes;
+// A bin of at most this many keys counts its gathered keys per key (32-bit
+// counts in the digit area, beside the candidates) and scans the counts for
+// x* instead of descending over the digits.
+constexpr int kHistKeys = 4096;
+static_assert(kHistKeys * sizeof(uint32_t) <= kDigitBytes, "the key counts sit in the digit area");
 // A thread adds at most this many tokens into a 32-bit slot (each at most
 // 2^22 + 1): up to ceil(V / (kPerVec * kNucThreads)) vectors of kPerVec and
 // one tail token, which kNucleusMaxVocab keeps within it.
@@ -259,6 +264,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   __shared__ int s_pick, s_over;
   __shared__ uint32_t s_klo, s_khi, s_prefix;
   __shared__ unsigned long long s_above, s_target;
+  __shared__ unsigned long long s_wsum[kNucWarps];
   grid_dependency_wait();
   grid_launch_dependents();
   const int g = blockIdx.x;
@@ -375,15 +381,9 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   const uint32_t klo = s_klo, range = s_khi - s_klo;
   uint32_t prefix = 0;   // the key offset of x* above the current level
   if (range > 0) {
-    // Gather the keys of the bin into this warp's segment. Each lane marks its
-    // logits in [x(klo), x(khi)] (a float test that takes every key of the
-    // range; a signed zero it takes beside them fails the descent's key test)
-    // in a bit mask per vector, and a warp prefix sum of the counts places
-    // them. The loop runs the same number of times in every lane of the warp
-    // (the shuffles need all 32).
-    TBits* seg = reinterpret_cast<TBits*>(reinterpret_cast<unsigned char*>(smem) + kDigitBytes) +
-                 warp * kSegKeys;
-    int cnt = 0;   // keys this warp found (uniform over the warp)
+    // Each lane marks its logits in [x(klo), x(khi)] (a float test that takes
+    // every key of the range; a signed zero it takes beside them fails the
+    // key test that follows) in a bit mask per vector.
     const uint32_t flo = key_bits<kKeyBits>(klo), fhi = key_bits<kKeyBits>(s_khi);
     // bit e set: logit e of the vector is in the range
     auto in_bits = [&](const uint4& v) -> uint32_t {
@@ -411,14 +411,26 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
     };
     // the fp32 bits of logit e of a vector
     auto logit_bits = [&](const uint4& v, int e) -> uint32_t {
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      const int k = sizeof(TBits) == 2 ? e >> 1 : e;   // the 32-bit word (selects, no local array)
+      const uint32_t x = k < 2 ? (k == 0 ? v.x : v.y) : (k == 2 ? v.z : v.w);
       if constexpr (sizeof(TBits) == 2) {
-        const uint32_t x = w[e >> 1];
         return (e & 1) ? (x & 0xFFFF0000u) : (x << 16);
       } else {
-        return w[e];
+        return x;
       }
     };
+    const bool narrow = range < static_cast<uint32_t>(kHistKeys);   // unsigned: an fp32 bin can span 2^31 keys
+    uint32_t* hist = smem;   // a narrow bin's count per key (the digit area)
+    if (narrow) {
+      for (int i = tid; i <= static_cast<int>(range); i += kNucThreads) hist[i] = 0u;
+      if (tid == 0) s_prefix = 0xFFFFFFFFu;
+    }
+    // Gather the keys of the bin into this warp's segment: a warp prefix sum
+    // of the lanes' counts places them. The loop runs the same number of times
+    // in every lane of the warp (the shuffles need all 32).
+    TBits* seg = reinterpret_cast<TBits*>(reinterpret_cast<unsigned char*>(smem) + kDigitBytes) +
+                 warp * kSegKeys;
+    int cnt = 0;   // keys this warp found (uniform over the warp)
     const int warp0 = tid - lane;
     for (int i0 = warp0; i0 < nvec; i0 += kNucUnroll * kNucThreads) {
       uint4 w[kNucUnroll];
@@ -467,6 +479,87 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
     const bool over = s_over != 0;
     const int n_mine = s_seg[warp];
 
+    if (narrow) {
+      // Stage 2, narrow bin: how many tokens hold each key of the bin (the
+      // tokens of one key share its logit and so its mass), counted over the
+      // gathered keys (over the row when a segment overflowed), then x* by a
+      // scan from the largest key down, each key's mass its count times the
+      // mass of its logit: the same integer sums as adding the tokens one by
+      // one. A lane holds the last key it met with its count so far and adds
+      // them when another key comes (or at the end): a row where one key holds
+      // most of the bin's tokens then makes few atomics on that key.
+      uint32_t run_key = 0xFFFFFFFFu, run_cnt = 0u;
+      auto count_d = [&](uint32_t d) {
+        if (d > range) return;
+        if (d != run_key) {
+          if (run_cnt != 0u) atomicAdd(hist + run_key, run_cnt);
+          run_key = d;
+          run_cnt = 0u;
+        }
+        ++run_cnt;
+      };
+      if (!over) {
+        for (int e = lane; e < n_mine; e += 32) count_d(static_cast<uint32_t>(seg[e]) - klo);
+      } else {
+        for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
+          for (uint32_t b = in_bits(v); b != 0u; b &= b - 1u)
+            count_d(logit_key<kKeyBits>(logit_bits(v, __ffs(b) - 1)) - klo);
+        });
+        for (int v = tail0 + tid; v < V; v += kNucThreads) count_d(logit_key<kKeyBits>(widen(row[v])) - klo);
+      }
+      if (run_cnt != 0u) atomicAdd(hist + run_key, run_cnt);
+      __syncthreads();
+      const int nk = static_cast<int>(range) + 1;
+      // key r from the top (r = 0 is key klo + range): its mass in the common unit
+      auto key_mass = [&](int r) -> unsigned long long {
+        const uint32_t c = hist[range - r];
+        if (c == 0u) return 0ull;
+        const uint32_t key = klo + range - static_cast<uint32_t>(r);
+        const uint32_t q = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk).q;
+        return to_common(static_cast<unsigned long long>(c) * q, jbin);
+      };
+      // Thread t takes the keys r in [t c, (t + 1) c): their mass, a block
+      // prefix sum over the threads in order, and the one thread whose keys
+      // hold the crossing of the target walks them.
+      const int chunk = (nk + kNucThreads - 1) / kNucThreads;
+      const int r0 = min(tid * chunk, nk), r1 = min(r0 + chunk, nk);
+      unsigned long long mine = 0;
+      for (int r = r0; r < r1; ++r) mine += key_mass(r);
+      unsigned long long incl = mine;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const unsigned long long t = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += t;
+      }
+      if (lane == 31) s_wsum[warp] = incl;
+      __syncthreads();
+      const unsigned long long target = s_target;
+      unsigned long long cum = s_above + (incl - mine);   // mass above this thread's first key
+      for (int w = 0; w < warp; ++w) cum += s_wsum[w];
+      if (cum < target && target <= cum + mine) {
+        for (int r = r0; r < r1; ++r) {
+          const unsigned long long h = key_mass(r);
+          if (cum + h >= target) {
+            s_prefix = range - static_cast<uint32_t>(r);
+            break;
+          }
+          cum += h;
+        }
+      }
+      __syncthreads();
+      const bool beyond = s_prefix == 0xFFFFFFFFu;   // the same in every thread
+      __syncthreads();
+      if (beyond) {   // the target is beyond the mass (truncation): keep down to the lowest key with mass
+        for (int r = r1 - 1; r >= r0; --r) {
+          if (hist[range - r] != 0u) {
+            atomicMin(&s_prefix, range - static_cast<uint32_t>(r));
+            break;
+          }
+        }
+        __syncthreads();
+      }
+      prefix = s_prefix == 0xFFFFFFFFu ? 0u : s_prefix;
+    } else {
     // Stage 2: the radix descent over d = key - klo, kDigitBits per level,
     // over the gathered keys (or the row, when a segment overflowed).
     const int nbits = 32 - __clz(range);
@@ -527,6 +620,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
       __syncthreads();
       prefix = s_prefix;
       above = s_above;
+    }
     }
   }
 

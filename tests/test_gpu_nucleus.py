@@ -207,3 +207,55 @@ def test_signed_zeros_at_the_boundary_are_kept_together(zb, dtype):
             zeros = rows[g] == 0.0
             assert kept[zeros].all() or not kept[zeros].any(), "the zeros split"
             assert _kept_ok(rows[g].astype(np.float64), kept, 1.0, top_p), (top_p, g)
+
+
+# The kernel's stage 2 counts the tokens of every key of the boundary bin and
+# scans the counts when the bin spans at most this many bf16 values, and
+# otherwise descends over the bin's keys by digits.
+HIST_KEYS = 4096
+
+
+def _bin_keys(x_row, T, top_p):
+    """How many bf16 values the boundary mass bin (one octave of probability
+    below the row maximum's, counted in whole octaves) spans."""
+    xs = nuc.kept_threshold(x_row, T, top_p)
+    m = float(np.max(x_row))
+    w = float(T) * np.log(2.0)
+    j = np.floor((m - xs) / w)
+    lo, hi = m - (j + 1) * w, m - j * w
+    allv = (np.arange(65536, dtype=np.uint32) << 16).view(np.float32)
+    allv = allv[np.isfinite(allv)]
+    return int(np.count_nonzero((allv > lo) & (allv <= hi)))
+
+
+@pytest.mark.parametrize("T", [0.3, 1.0])
+def test_kept_sets_on_both_stage2_paths_with_heavy_ties(zb, T):
+    """bf16 rows of the decode vocabulary whose boundary bin is narrow (the
+    key counts: one key holding nearly every token and two adjacent keys
+    interleaved, both overflowing the gathered segments, and a normal spread)
+    or crosses zero (tens of thousands of keys: the digit descent)."""
+    rng = np.random.default_rng(29)
+    V = 151936
+    peaks = rng.choice(V, 40, replace=False)
+    one_key = np.full(V, 1.25, dtype=np.float32)
+    one_key[peaks] = 4.0
+    two_keys = np.where(rng.random(V) < 0.5, 1.5, 1.5078125).astype(np.float32)
+    two_keys[peaks] = 4.0
+    spread = rng.normal(size=V).astype(np.float32)
+    near_zero = rng.uniform(-0.3, 0.3, V).astype(np.float32)
+    near_zero[peaks[:5]] = 0.4
+    x = pen.bf16_round(np.stack([one_key, two_keys, spread, near_zero]))
+    for top_p in (0.3, 0.9, 0.999):
+        logits, _, _ = _run(zb, x, torch.bfloat16, [0, 4], T, top_p)
+        got = logits.float().cpu().numpy()
+        for g in range(4):
+            xg = x[g].astype(np.float64)
+            keys = _bin_keys(xg, T, top_p)
+            if g == 3 and T == 1.0 and top_p < 0.99:
+                assert keys > HIST_KEYS, keys          # the digit descent
+            elif g < 3:
+                assert keys < HIST_KEYS // 2, keys     # the key counts
+            kept = np.isfinite(got[g])
+            assert np.array_equal(got[g][kept], x[g][kept])
+            assert (got[g][~kept] == -np.inf).all()
+            assert _kept_ok(xg, kept, T, top_p), (T, top_p, g)
