@@ -132,8 +132,17 @@ struct Mass {
   uint32_t q;   // 0 for a massless token (a <= -42, or NaN)
   uint32_t j;
 };
-__device__ __forceinline__ Mass token_mass(float x, float k2, float neg_mk) {
-  const float a = fmaf(x, k2, neg_mk);
+// The exponent argument a = (x - m) k2: the difference is exact for every
+// token with mass once |m| is large (x within a factor of two of m), and
+// only the product rounds; x k2 - m k2 would carry the rounding of m k2, up
+// to 2^-25 |m k2|, into every token's argument and lift the tokens nearest
+// the maximum above 0. It is monotone in x, so each bin is a range of keys.
+__device__ __forceinline__ float mass_arg(float x, float m, float k2) {
+  return __fmul_rn(__fsub_rn(x, m), k2);
+}
+
+__device__ __forceinline__ Mass token_mass(float x, float k2, float m) {
+  const float a = mass_arg(x, m, k2);
   const float c = a > kMassFloor ? fminf(a, 0.f) : -INFINITY;   // -inf: e = 0
   const uint32_t j =
       __float_as_uint(__fmaf_rz(fmaxf(c, kMassFloorUp), -1.f, kBinMagic)) - kBinMagicBits;
@@ -145,9 +154,9 @@ __device__ __forceinline__ Mass token_mass(float x, float k2, float neg_mk) {
 // token_mass for two logits at once: the same operations, the ones with a
 // paired fp32 form taken two at a time (each half rounds exactly as the
 // scalar instruction does), so each result is token_mass's bit for bit.
-__device__ __forceinline__ void token_mass2(float x0, float x1, float k2, float neg_mk, Mass& s0,
+__device__ __forceinline__ void token_mass2(float x0, float x1, float k2, float m, Mass& s0,
                                             Mass& s1) {
-  const float2 a = __ffma2_rn(make_float2(x0, x1), make_float2(k2, k2), make_float2(neg_mk, neg_mk));
+  const float2 a = __fmul2_rn(__fadd2_rn(make_float2(x0, x1), make_float2(-m, -m)), make_float2(k2, k2));
   const float c0 = a.x > kMassFloor ? fminf(a.x, 0.f) : -INFINITY;
   const float c1 = a.y > kMassFloor ? fminf(a.y, 0.f) : -INFINITY;
   const float2 y = __ffma2_rz(make_float2(fmaxf(c0, kMassFloorUp), fmaxf(c1, kMassFloorUp)),
@@ -163,8 +172,8 @@ __device__ __forceinline__ void token_mass2(float x0, float x1, float k2, float 
 }
 
 // The bin of a logit (kMassBins for a massless one): token_mass's bin test.
-__device__ __forceinline__ int token_bin(float x, float k2, float neg_mk) {
-  const float a = fmaf(x, k2, neg_mk);
+__device__ __forceinline__ int token_bin(float x, float k2, float m) {
+  const float a = mass_arg(x, m, k2);
   if (!(a > kMassFloor)) return kMassBins;
   const float c = fminf(fmaxf(a, kMassFloorUp), 0.f);
   return static_cast<int>(__float_as_uint(__fmaf_rz(c, -1.f, kBinMagic)) - kBinMagicBits);
@@ -300,7 +309,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   m = s_max[0];
   for (int w = 1; w < kNucWarps; ++w) m = fmaxf(m, s_max[w]);
   if (!(m > -INFINITY)) return;   // every logit -inf (or NaN): nothing to cut
-  const float k2 = a.k2, neg_mk = -m * a.k2;
+  const float k2 = a.k2;
 
   // Stage 1: the mass bins in private slots. A slot has one writer, so its
   // updates are shared-memory reductions (no load-add-store chain from one
@@ -310,13 +319,13 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   for (int j = 0; j < kMassBins; ++j) own[j * kNucThreads] = 0u;
   auto add_mass2 = [&](uint32_t f0, uint32_t f1) {
     Mass s0, s1;
-    token_mass2(__uint_as_float(f0), __uint_as_float(f1), k2, neg_mk, s0, s1);
+    token_mass2(__uint_as_float(f0), __uint_as_float(f1), k2, m, s0, s1);
     atomicAdd(own + s0.j * kNucThreads, s0.q);
     atomicAdd(own + s1.j * kNucThreads, s1.q);
   };
   for_each_vec(row4, nvec, tid, [&](const uint4& v, int) { each_logit_pair<TBits>(v, add_mass2); });
   for (int v = tail0 + tid; v < V; v += kNucThreads) {
-    const Mass s = token_mass(__uint_as_float(widen(row[v])), k2, neg_mk);
+    const Mass s = token_mass(__uint_as_float(widen(row[v])), k2, m);
     atomicAdd(own + s.j * kNucThreads, s.q);
   }
   __syncthreads();
@@ -368,7 +377,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   if (warp == 0) {
     const uint32_t lo = logit_key<kKeyBits>(0xFF800000u), hi = logit_key<kKeyBits>(0x7F800000u);
     auto bin_of = [&](uint32_t key) {
-      return token_bin(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk);
+      return token_bin(__uint_as_float(key_bits<kKeyBits>(key)), k2, m);
     };
     const uint32_t klo = first_true_key(lo, hi, lane, [&](uint32_t k) { return bin_of(k) <= jbin; });
     const uint32_t kend = first_true_key(lo, hi, lane, [&](uint32_t k) { return bin_of(k) < jbin; });
@@ -455,8 +464,8 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
       int pos = cnt + incl - c;
 #pragma unroll
       for (int u = 0; u < kNucUnroll; ++u) {
-        for (uint32_t m = bits[u]; m != 0u; m &= m - 1u, ++pos) {
-          const int e = __ffs(m) - 1;
+        for (uint32_t mb = bits[u]; mb != 0u; mb &= mb - 1u, ++pos) {
+          const int e = __ffs(mb) - 1;
           if (pos < kSegKeys) seg[pos] = static_cast<TBits>(logit_key<kKeyBits>(logit_bits(w[u], e)));
         }
       }
@@ -515,7 +524,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
         const uint32_t c = hist[range - r];
         if (c == 0u) return 0ull;
         const uint32_t key = klo + range - static_cast<uint32_t>(r);
-        const uint32_t q = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk).q;
+        const uint32_t q = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, m).q;
         return to_common(static_cast<unsigned long long>(c) * q, jbin);
       };
       // Thread t takes the keys r in [t c, (t + 1) c): their mass, a block
@@ -574,7 +583,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
         const uint32_t d = key - klo;
         if (d > range) return;
         if (level > 0 && (d >> (shift + kDigitBits)) != prefix) return;
-        const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, neg_mk);
+        const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, m);
         atomicAdd(own + ((d >> shift) & (kDigits - 1)) * kNucThreads, s.q);
       };
       if (!over) {

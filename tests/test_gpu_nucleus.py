@@ -210,22 +210,35 @@ def test_signed_zeros_at_the_boundary_are_kept_together(zb, dtype):
 
 
 # The kernel's stage 2 counts the tokens of every key of the boundary bin and
-# scans the counts when the bin spans at most this many bf16 values, and
-# otherwise descends over the bin's keys by digits.
+# scans the counts when the bin spans at most this many logit values (bf16 or
+# fp32), and otherwise descends over the bin's keys by digits.
 HIST_KEYS = 4096
 
 
-def _bin_keys(x_row, T, top_p):
-    """How many bf16 values the boundary mass bin (one octave of probability
-    below the row maximum's, counted in whole octaves) spans."""
+def _bin_keys(x_row, T, top_p, dtype=torch.bfloat16):
+    """How many representable logit values (bf16 or fp32) the boundary mass
+    bin (one octave of probability below the row maximum's, counted in whole
+    octaves) spans."""
     xs = nuc.kept_threshold(x_row, T, top_p)
     m = float(np.max(x_row))
     w = float(T) * np.log(2.0)
     j = np.floor((m - xs) / w)
     lo, hi = m - (j + 1) * w, m - j * w
-    allv = (np.arange(65536, dtype=np.uint32) << 16).view(np.float32)
-    allv = allv[np.isfinite(allv)]
-    return int(np.count_nonzero((allv > lo) & (allv <= hi)))
+    if dtype == torch.bfloat16:
+        allv = (np.arange(65536, dtype=np.uint32) << 16).view(np.float32)
+        allv = allv[np.isfinite(allv)]
+        return int(np.count_nonzero((allv > lo) & (allv <= hi)))
+
+    def key(v):   # order-preserving key of an fp32 value
+        b = int(np.array([v], dtype=np.float32).view(np.uint32)[0])
+        return b ^ 0xFFFFFFFF if b & 0x80000000 else b | 0x80000000
+
+    lo32, hi32 = np.float32(lo), np.float32(hi)
+    if lo32 <= lo:   # the smallest fp32 value above lo
+        lo32 = np.nextafter(lo32, np.float32(np.inf))
+    if hi32 > hi:
+        hi32 = np.nextafter(hi32, np.float32(-np.inf))
+    return key(hi32) - key(lo32) + 1
 
 
 @pytest.mark.parametrize("T", [0.3, 1.0])
@@ -255,6 +268,33 @@ def test_kept_sets_on_both_stage2_paths_with_heavy_ties(zb, T):
                 assert keys > HIST_KEYS, keys          # the digit descent
             elif g < 3:
                 assert keys < HIST_KEYS // 2, keys     # the key counts
+            kept = np.isfinite(got[g])
+            assert np.array_equal(got[g][kept], x[g][kept])
+            assert (got[g][~kept] == -np.inf).all()
+            assert _kept_ok(xg, kept, T, top_p), (T, top_p, g)
+
+
+def test_kept_sets_on_the_key_counts_with_fp32_logits(zb):
+    """fp32 rows far from zero, where one octave of probability spans a few
+    hundred fp32 values: the key counts with 32-bit keys (a spread, a plateau
+    with peaks), beside a row near zero that takes the digit descent."""
+    rng = np.random.default_rng(31)
+    V = 20000
+    spread = (20000.0 + rng.normal(scale=2.0, size=V)).astype(np.float32)
+    plateau = np.full(V, 20000.0, dtype=np.float32)
+    plateau[rng.choice(V, 30, replace=False)] = 20003.0
+    near_zero = rng.normal(scale=0.5, size=V).astype(np.float32)
+    x = np.stack([spread, plateau, near_zero])
+    for T, top_p in ((1.0, 0.5), (1.0, 0.9), (0.7, 0.99)):
+        logits, _, _ = _run(zb, x, torch.float32, [0, 3], T, top_p)
+        got = logits.cpu().numpy()
+        for g in range(3):
+            xg = x[g].astype(np.float64)
+            keys = _bin_keys(xg, T, top_p, torch.float32)
+            if g < 2:
+                assert keys < HIST_KEYS // 2, keys     # the key counts
+            else:
+                assert keys > HIST_KEYS, keys          # the digit descent
             kept = np.isfinite(got[g])
             assert np.array_equal(got[g][kept], x[g][kept])
             assert (got[g][~kept] == -np.inf).all()
