@@ -569,67 +569,67 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
       }
       prefix = s_prefix == 0xFFFFFFFFu ? 0u : s_prefix;
     } else {
-    // Stage 2: the radix descent over d = key - klo, kDigitBits per level,
-    // over the gathered keys (or the row, when a segment overflowed).
-    const int nbits = 32 - __clz(range);
-    const int levels = (nbits + kDigitBits - 1) / kDigitBits;
-    const unsigned long long target = s_target;
-    unsigned long long above = s_above;   // mass of the tokens above the current range
-    for (int level = 0; level < levels; ++level) {
-      const int shift = kDigitBits * (levels - 1 - level);
+      // Stage 2, wide bin: the radix descent over d = key - klo, kDigitBits per
+      // level, over the gathered keys (or the row, when a segment overflowed).
+      const int nbits = 32 - __clz(range);
+      const int levels = (nbits + kDigitBits - 1) / kDigitBits;
+      const unsigned long long target = s_target;
+      unsigned long long above = s_above;   // mass of the tokens above the current range
+      for (int level = 0; level < levels; ++level) {
+        const int shift = kDigitBits * (levels - 1 - level);
 #pragma unroll
-      for (int k = 0; k < kDigits; ++k) own[k * kNucThreads] = 0u;
-      auto add = [&](uint32_t key) {
-        const uint32_t d = key - klo;
-        if (d > range) return;
-        if (level > 0 && (d >> (shift + kDigitBits)) != prefix) return;
-        const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, m);
-        atomicAdd(own + ((d >> shift) & (kDigits - 1)) * kNucThreads, s.q);
-      };
-      if (!over) {
-        for (int e = lane; e < n_mine; e += 32) add(seg[e]);
-      } else {
-        for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
-          each_logit<TBits>(v, [&](uint32_t f) { add(logit_key<kKeyBits>(f)); });
-        });
-        for (int v = tail0 + tid; v < V; v += kNucThreads) add(logit_key<kKeyBits>(widen(row[v])));
-      }
-      __syncthreads();
-      if (warp < kDigits) {   // digit `warp`'s total, in a fixed order
-        unsigned long long t = 0;
-        for (int i = lane; i < kNucThreads; i += 32) t += smem[warp * kNucThreads + i];
+        for (int k = 0; k < kDigits; ++k) own[k * kNucThreads] = 0u;
+        auto add = [&](uint32_t key) {
+          const uint32_t d = key - klo;
+          if (d > range) return;
+          if (level > 0 && (d >> (shift + kDigitBits)) != prefix) return;
+          const Mass s = token_mass(__uint_as_float(key_bits<kKeyBits>(key)), k2, m);
+          atomicAdd(own + ((d >> shift) & (kDigits - 1)) * kNucThreads, s.q);
+        };
+        if (!over) {
+          for (int e = lane; e < n_mine; e += 32) add(seg[e]);
+        } else {
+          for_each_vec(row4, nvec, tid, [&](const uint4& v, int) {
+            each_logit<TBits>(v, [&](uint32_t f) { add(logit_key<kKeyBits>(f)); });
+          });
+          for (int v = tail0 + tid; v < V; v += kNucThreads) add(logit_key<kKeyBits>(widen(row[v])));
+        }
+        __syncthreads();
+        if (warp < kDigits) {   // digit `warp`'s total, in a fixed order
+          unsigned long long t = 0;
+          for (int i = lane; i < kNucThreads; i += 32) t += smem[warp * kNucThreads + i];
 #pragma unroll
-        for (int d = 16; d >= 1; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
-        if (lane == 0) bins[warp] = t;
-      }
-      __syncthreads();
-      if (tid == 0) {
-        unsigned long long cum = above;
-        int pick = -1, lowest = -1;
+          for (int d = 16; d >= 1; d >>= 1) t += __shfl_xor_sync(0xffffffffu, t, d);
+          if (lane == 0) bins[warp] = t;
+        }
+        __syncthreads();
+        if (tid == 0) {
+          unsigned long long cum = above;
+          int pick = -1, lowest = -1;
 #pragma unroll 1
-        for (int k = kDigits - 1; k >= 0; --k) {
-          if (bins[k] == 0ull) continue;
-          const unsigned long long h = to_common(bins[k], jbin);
-          lowest = k;
-          if (cum + h >= target) {
-            pick = k;
-            break;
+          for (int k = kDigits - 1; k >= 0; --k) {
+            if (bins[k] == 0ull) continue;
+            const unsigned long long h = to_common(bins[k], jbin);
+            lowest = k;
+            if (cum + h >= target) {
+              pick = k;
+              break;
+            }
+            cum += h;
           }
-          cum += h;
-        }
-        if (pick < 0) {   // the target is beyond the mass (truncation): keep down to the lowest digit
-          pick = lowest < 0 ? 0 : lowest;
-          cum = above;
+          if (pick < 0) {   // the target is beyond the mass (truncation): keep down to the lowest digit
+            pick = lowest < 0 ? 0 : lowest;
+            cum = above;
 #pragma unroll 1
-          for (int k = kDigits - 1; k > pick; --k) cum += to_common(bins[k], jbin);
+            for (int k = kDigits - 1; k > pick; --k) cum += to_common(bins[k], jbin);
+          }
+          s_prefix = (prefix << kDigitBits) | static_cast<uint32_t>(pick);
+          s_above = cum;
         }
-        s_prefix = (prefix << kDigitBits) | static_cast<uint32_t>(pick);
-        s_above = cum;
+        __syncthreads();
+        prefix = s_prefix;
+        above = s_above;
       }
-      __syncthreads();
-      prefix = s_prefix;
-      above = s_above;
-    }
     }
   }
 
