@@ -157,8 +157,10 @@ __device__ __forceinline__ Mass token_mass(float x, float k2, float m) {
 __device__ __forceinline__ void token_mass2(float x0, float x1, float k2, float m, Mass& s0,
                                             Mass& s1) {
   const float2 a = __fmul2_rn(__fadd2_rn(make_float2(x0, x1), make_float2(-m, -m)), make_float2(k2, k2));
-  const float c0 = a.x > kMassFloor ? fminf(a.x, 0.f) : -INFINITY;
-  const float c1 = a.y > kMassFloor ? fminf(a.y, 0.f) : -INFINITY;
+  // a <= 0 for every token of the row (x <= m): token_mass's clamp at 0 is
+  // the identity here (a signed zero gives the same bin and mass either way)
+  const float c0 = a.x > kMassFloor ? a.x : -INFINITY;
+  const float c1 = a.y > kMassFloor ? a.y : -INFINITY;
   const float2 y = __ffma2_rz(make_float2(fmaxf(c0, kMassFloorUp), fmaxf(c1, kMassFloorUp)),
                               make_float2(-1.f, -1.f), make_float2(kBinMagic, kBinMagic));
   s0.j = __float_as_uint(y.x) - kBinMagicBits;
@@ -373,7 +375,9 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
   if (jbin < 0) return;   // no token has mass (a +inf logit): nothing to cut
 
   // The key range of bin jbin (the bin falls as the key grows; NaN keys lie
-  // outside [key(-inf), key(+inf)]).
+  // outside [key(-inf), key(+inf)]), cut at the maximum: no token lies above
+  // it, and bin 0 would otherwise reach to +inf (one past the maximum's key,
+  // so that +0 stays inside when the maximum came out as -0).
   if (warp == 0) {
     const uint32_t lo = logit_key<kKeyBits>(0xFF800000u), hi = logit_key<kKeyBits>(0x7F800000u);
     auto bin_of = [&](uint32_t key) {
@@ -383,7 +387,7 @@ __global__ void __launch_bounds__(kNucThreads, 2) nucleus_kernel(const NucleusPa
     const uint32_t kend = first_true_key(lo, hi, lane, [&](uint32_t k) { return bin_of(k) < jbin; });
     if (lane == 0) {
       s_klo = klo;
-      s_khi = kend - 1;
+      s_khi = min(kend - 1, logit_key<kKeyBits>(__float_as_uint(m)) + 1u);
     }
   }
   __syncthreads();
