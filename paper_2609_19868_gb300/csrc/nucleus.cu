@@ -132,11 +132,12 @@ struct Mass {
   uint32_t q;   // 0 for a massless token (a <= -42, or NaN)
   uint32_t j;
 };
-// The exponent argument a = (x - m) k2: the difference is exact for every
-// token with mass once |m| is large (x within a factor of two of m), and
-// only the product rounds; x k2 - m k2 would carry the rounding of m k2, up
-// to 2^-25 |m k2|, into every token's argument and lift the tokens nearest
-// the maximum above 0. It is monotone in x, so each bin is a range of keys.
+// The exponent argument a = (x - m) k2: the difference and the product each
+// round within 2^-24 of their own value, so a is within 2^-23 |a| of exact
+// (the heavy tokens near a = 0 nearly exact); x k2 - m k2 would carry the
+// rounding of m k2, up to 2^-25 |m k2| whatever a is, into every token's
+// argument and lift the tokens nearest the maximum above 0. It is monotone
+// in x, so each bin is a range of keys.
 __device__ __forceinline__ float mass_arg(float x, float m, float k2) {
   return __fmul_rn(__fsub_rn(x, m), k2);
 }
