@@ -1098,12 +1098,17 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
 // suffices: each group rescales and finishes columns [64g, 64g + 64) of it,
 // and the groups' row sums add at the end. The key range is not split (one
 // CTA per pair).
-constexpr int kPairStagesK = 3;
+constexpr int kPairStagesK = 2;
 constexpr int kPairStagesV = 2;
 constexpr uint32_t kPOffQ = 0;                                   // Q_A, then Q_B
 constexpr uint32_t kPOffK = 2 * kTileBytes;
 constexpr uint32_t kPOffV = kPOffK + kPairStagesK * kTileBytes;
-constexpr uint32_t kPOffBar = kPOffV + kPairStagesV * kTileBytes;
+// The row maxima the two softmax warps of a row trade each job,
+// [job parity][group][row]: one buffer per parity, so a warp's write for job
+// j + 2 comes after barrier j + 1, which the other warp reaches only once it
+// has read job j's value.
+constexpr uint32_t kPOffX = kPOffV + kPairStagesV * kTileBytes;
+constexpr uint32_t kPOffBar = kPOffX + 2 * 2 * 128 * sizeof(float);
 
 struct PairBars {
   uint64_t q_full;
@@ -1133,6 +1138,7 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   PairBars* bars = reinterpret_cast<PairBars*>(smem + kPOffBar);
+  float* xmax = reinterpret_cast<float*>(smem + kPOffX);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -1377,8 +1383,8 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
       const int c0 = c_tile + grp * 64;   // this group's keys
       if (ok) ok = wait_bar(&bars->s_full[j & 1], (j >> 1) & 1, bars, p);
       ok = __all_sync(0xffffffffu, ok);
-      // This group's scores and their row maximum, which it leaves in column
-      // 32 of its half of S (a column that neither P nor P*V uses).
+      // This group's scores and their row maximum, which it leaves in shared
+      // memory for the other group of the row.
       float s[64];
       float mx = -INFINITY;
       if (ok) {
@@ -1386,14 +1392,13 @@ slot_attn_pair_kernel(const __grid_constant__ CUtensorMap map_q,
         tmem_ld_32x32b_x64(t_s + grp * 64, s);
         mask64(s, c0, limit, hide_hi);
         mx = max64(s);
-        tmem_st_32x32b_x1(t_s + grp * 64 + 32, mx);
-        tc_fence_before();
+        xmax[((j & 1) * 2 + grp) * 128 + m] = mx;
       }
       // Both warps of the quadrant arrive here every job and leave together,
-      // going on only if both got their S; then each reads the other's maximum.
+      // going on only if both got their S; the barrier orders their shared-
+      // memory writes before the reads, and each reads the other's maximum.
       if (!named_bar_and(2 + wq, 64, ok)) { ok = false; break; }
-      tc_fence_after();
-      mx = fmaxf(mx, tmem_ld_32x32b_x1(t_s + (1 - grp) * 64 + 32));
+      mx = fmaxf(mx, xmax[((j & 1) * 2 + (1 - grp)) * 128 + m]);
       float m_run = t ? m_runB : m_runA;
       float l_run = t ? l_runB : l_runA;
       const float m_new = fmaxf(m_run, mx * sl2);
