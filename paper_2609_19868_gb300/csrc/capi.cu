@@ -129,15 +129,10 @@ Plan plan_tc(const zarya_attn_desc* d, int sms) {
   const int tiles = static_cast<int>((kv_max + kBlockN - 1) / kBlockN);
   // Paged caches cost one tensor copy per page per tile; serving two M-tiles
   // of a (sequence, KV head) from each tile halves the copies per unit of
-  // work. Taken when the pairs alone fill the GPU (no key split needed); for
-  // a contiguous cache, when they fill it three times over, so that the
-  // longest-first order can even out their lengths (a ragged batch of 512
-  // pairs ran 1.4 % faster than the single-tile kernel with key splits; 256
-  // pairs of long sequences would leave a ragged last wave).
+  // work. Taken when the pairs alone fill the GPU (no key split needed).
   const long long pairs = (p.m_tiles + 1) / 2;
-  const long long pair_items = static_cast<long long>(d->batch) * d->n_kv_heads * pairs;
-  if (d->kv_splits == 0 && p.m_tiles >= 2 &&
-      ((d->page_size > 0 && pair_items >= sms) || pair_items >= 3LL * sms)) {
+  if (d->page_size > 0 && d->kv_splits == 0 && p.m_tiles >= 2 &&
+      static_cast<long long>(d->batch) * d->n_kv_heads * pairs >= sms) {
     p.pair = 1;
     p.splits = 1;
     return with_schedule(p, d, sms);
