@@ -1093,8 +1093,8 @@ slot_attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
 //
 // Both softmax groups work on every job: group g takes keys [64g, 64g + 64)
 // of the tile, but the two share the row maximum (each leaves its half's
-// maximum in a spare TMEM column of its half, the quadrant's two warps meet
-// at a named barrier, and each reads the other's), so one O per M-tile
+// maximum in a shared-memory buffer of the job's parity, the quadrant's two
+// warps meet at a named barrier, and each reads the other's), so one O per M-tile
 // suffices: each group rescales and finishes columns [64g, 64g + 64) of it,
 // and the groups' row sums add at the end. The key range is not split (one
 // CTA per pair).
